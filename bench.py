@@ -1,0 +1,503 @@
+#!/usr/bin/env python3
+"""Benchmark of the fused AutoLoCo outer-sync round on GB300.
+
+A step is one outer synchronisation round (Algorithm 1: pseudo-gradients,
+average, D_t / C_t, corrected Nesterov step, replica reset) over one batch
+of synthetic worker endpoints, called through the C ABI.  The default
+workload is the Llama-style 150M parameter set (12 layers, d 768, tied
+embeddings; N = 137,841,408) with 8 fp32 worker replicas and consecutive
+rounds whose horizons are drawn by seed from {50, 100, 150, 200, 300},
+momentum carried across rounds.
+
+Between timed rounds the replicas are refilled with new endpoints (this
+stands in for the workers' inner loops and is not timed); each round is
+bracketed by CUDA events on the launch stream, and the whole loop by a
+barrier and device synchronisation.  Every round reads and writes
+11 GB, far more than the 129 MB L2, so no L2 flush is needed.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 oracle on the host
+
+Multi-GPU: the round does not shard across GPUs; with N > 1 every rank runs
+an independent replica of the workload on its own GPU ("replicas only") and
+the value is the total rounds/s of the job.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = ("outer-sync rounds/s and achieved HBM GB/s (fraction of GB300 "
+          "roofline) at N params × M workers")
+UNIT = "rounds/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+KERNEL_NAME = "sync_kernel"
+
+
+def workloads_by_name():
+    from paper_2609_36662_gb300 import workloads as W
+    out = {w.name: w for w in W.all_configs()}
+    return out
+
+
+def parse_flat(name: str):
+    """flat<N>_m<M>_<f32|bf16>: a flat vector of N parameters (used for the
+    small profiling cases)."""
+    import re
+    from paper_2609_36662_gb300 import workloads as W
+    m = re.fullmatch(r"flat(\d+)_m(\d+)_(f32|bf16)", name)
+    if not m:
+        return None
+    return W.small(int(m.group(1)), int(m.group(2)), m.group(3), seed=4,
+                   H_sel=200, H_base=100)
+
+
+def default_workload_name():
+    from paper_2609_36662_gb300 import workloads as W
+    return W.llama_150m().name
+
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_36662_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the fused pass from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except Exception:
+        return None
+    entry = rec.get(workload)
+    if not entry or entry.get("kernel_hash") != kernel_source_hash():
+        return None
+    return entry.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed
+    region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        time.sleep(0.2)
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), parts[4:8]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, flags in rows
+                          for i, f in enumerate(flags) if f.lower() == "active"})
+        mx = max(r[1] for r in rows)
+        loaded = [r[0] for r in rows if r[0] >= 0.5 * mx] or [r[0] for r in rows]
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------- distributed
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def reduce_max(value: float, world: int, device=None) -> float:
+    """Max over ranks (identity for one rank)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64,
+                     device=device if device is not None else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(units_per_rank: float, seconds_max: float, world: int) -> float:
+    """Whole-job throughput: the units every rank processed over the slowest
+    rank's time."""
+    return units_per_rank * world / seconds_max
+
+
+# ------------------------------------------------------------ CPU oracle
+
+def oracle_sample(w, g, v, xs, elems: int, step: int, H_sel: int):
+    """Time the oracle (single thread, as it stands) on the first `elems`
+    elements of the round.  Returns seconds."""
+    import numpy as np
+    import torch
+    import oracle as O
+    n = min(elems, w.numel)
+    gh = g[:n].cpu().numpy()
+    vh = v[:n].cpu().numpy()
+    if w.dtype == "f32":
+        xh = [x[:n].cpu().numpy() for x in xs]
+    else:
+        xh = [x[:n].cpu().view(torch.int16).numpy().view(np.uint16)
+              for x in xs]
+    s = w.schedule
+    sched = O.Schedule(s.kind, s.peak_lr, s.final_lr, s.warmup_steps,
+                       s.total_steps)
+    t0 = time.perf_counter()
+    O.sync_round(gh, vh, xh, O.F32 if w.dtype == "f32" else O.BF16, sched,
+                 step, H_sel, w.H_base, w.outer_lr, w.outer_beta)
+    return time.perf_counter() - t0, n
+
+
+def calibrated_sample(w, g, v, xs, step, H_sel, target_s):
+    """Pick a sample size whose oracle run takes about target_s seconds."""
+    probe = min(w.numel, 1 << 20)
+    t, n = oracle_sample(w, g, v, xs, probe, step, H_sel)
+    per_elem = t / n
+    want = int(target_s / max(per_elem, 1e-12))
+    want = max(1 << 16, min(w.numel, want))
+    return want
+
+
+# ------------------------------------------------------------- main arms
+
+def run_reference(args, w):
+    """The fp64 oracle on the host cores, timed per step on a bounded
+    sample of the workload (rank 0 only)."""
+    import torch
+    from paper_2609_36662_gb300 import workloads as W
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    g = W.make_global(w, "cpu")
+    v = W.make_momentum(w, "cpu")
+    rounds = W.steps_of_rounds(w, args.warmup + args.steps)
+    step0, h0 = rounds[0]
+
+    def endpoints(n_chunks):
+        n = min(w.numel, n_chunks * W.CHUNK)
+        xs = [torch.empty(n, dtype=W.replica_dtype(w)) for _ in range(w.M)]
+        W.fill_replicas(w, g[:n], xs, 0, 0, n_chunks)
+        return xs
+
+    # calibrate on the first chunk, then draw only the chunks the sample needs
+    xs = endpoints(1)
+    sample = calibrated_sample(w, g, v, xs, step0, h0, args.ref_step_seconds)
+    need = (sample + W.CHUNK - 1) // W.CHUNK
+    if need > 1:
+        xs = endpoints(need)
+    times = []
+    for k, (step, hsel) in enumerate(rounds):
+        t, n = oracle_sample(w, g, v, xs, sample, step, hsel)
+        if k >= args.warmup:
+            times.append(t)
+    sec_per_round = statistics.mean(times) * w.numel / sample
+    value = 1.0 / sec_per_round
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": sec_per_round * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": config_block(w),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1,
+                         "kind": "oracle",
+                         "sample": f"first {sample} of {w.numel} parameters "
+                                   f"x {w.M} workers per step, scaled to a "
+                                   f"full round"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_block(w):
+    from paper_2609_36662_gb300 import workloads as W
+    return {"workload": w.name, "N": w.numel, "M": w.M,
+            "replica_dtype": w.dtype, "outer_state_dtype": "f32",
+            "shape": (None if w.shape is None else
+                      {"layers": w.shape.layers, "d_model": w.shape.d_model,
+                       "heads": w.shape.heads, "kv_heads": w.shape.kv_heads,
+                       "ffn": w.shape.ffn, "vocab": w.shape.vocab,
+                       "tied": w.shape.tied}),
+            "bytes_per_round": w.bytes_per_round(),
+            "l2": f"no flush: each round moves {w.bytes_per_round() / 1e9:.1f} GB "
+                  "> 129 MB L2",
+            "H_base": w.H_base, "start_step": w.start_step,
+            "parallelism": "replicas only"}
+
+
+def run_cuda(args, w):
+    import numpy as np
+    import torch
+    from paper_2609_36662_gb300 import aloco as A
+    from paper_2609_36662_gb300 import workloads as W
+
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", torch.cuda.current_device())
+    A.load()
+
+    rounds = W.steps_of_rounds(w, args.warmup + args.steps)
+    g = W.make_global(w, device)
+    v = W.make_momentum(w, device)
+    xs = W.fill_replicas(w, g, W.alloc_replicas(w, device), 0)
+    s = w.schedule
+    sched = A.Schedule.make(s.kind, s.peak_lr, s.final_lr, s.warmup_steps,
+                            s.total_steps)
+    stream = torch.cuda.Stream(device)
+
+    # CPU baseline: the oracle on a bounded sample of round 0 (rank 0, N=1)
+    cpu_baseline = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        step0, h0 = rounds[0]
+        sample = calibrated_sample(w, g, v, xs, step0, h0, args.cpu_seconds)
+        t, n = oracle_sample(w, g, v, xs, sample, step0, h0)
+        cpu_baseline = {"value": (n / w.numel) / t, "unit": UNIT, "cores": 1,
+                        "kind": "oracle",
+                        "sample": f"first {n} of {w.numel} parameters x "
+                                  f"{w.M} workers of one round "
+                                  f"({t:.1f} s), scaled to a full round"}
+
+    opts = A.default_opts(time_kernel=1)
+    step_ms, kern_ms, statuses = [], [], []
+    ev = [(torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in rounds]
+
+    def one_round(k):
+        step, hsel = rounds[k]
+        if k > 0:
+            with torch.cuda.stream(stream):
+                W.fill_replicas(w, g, xs, k)      # untimed: the inner loops
+        ev[k][0].record(stream)
+        st = A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step,
+                    schedule=sched, outer_lr=w.outer_lr,
+                    outer_beta=w.outer_beta, opts=opts, stream=stream)
+        ev[k][1].record(stream)
+        return st
+
+    for k in range(args.warmup):
+        one_round(k)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter()
+    with ClockSampler(device.index) as clocks:
+        for k in range(args.warmup, args.warmup + args.steps):
+            st = one_round(k)
+            statuses.append(st["status"])
+            kern_ms.append(st["kernel_ms"])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter() - t_wall
+    for k in range(args.warmup, args.warmup + args.steps):
+        step_ms.append(ev[k][0].elapsed_time(ev[k][1]))
+
+    ms_step = statistics.mean(step_ms)
+    ms_step = reduce_max(ms_step, world, device)
+    ms_kern = reduce_max(statistics.mean(kern_ms), world, device)
+    value = job_value(1.0, ms_step / 1e3, world)
+    peak, peak_kind = hbm_peak()
+    achieved = w.bytes_per_round() / (ms_kern / 1e3) / 1e9
+
+    # end to end through the C ABI with host buffers: H2D of the round's
+    # inputs from pinned memory, the round, D2H of theta' and v'
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded; Llama-shaped parameter set, "
+                    "shared/private drift noise)",
+            "config": config_block(w),
+            "rounds_per_s_per_gpu": 1e3 / ms_step,
+            "elem_per_s": value * w.numel * w.M,
+            "kernel_ms": ms_kern,
+            "hbm_gbs": achieved,
+            "frac_of_nominal_8000": achieved / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak,
+                         "peak_source": peak_kind,
+                         "traffic": recorded_traffic(w.name),
+                         "kernel": KERNEL_NAME,
+                         "algorithmic_bytes_per_launch": w.bytes_per_round()},
+            "cpu_baseline": cpu_baseline,
+            "e2e": e2e,
+            "gpu_launches": args.steps,
+            "clocks": clocks.summary(),
+            "status_ok": all(s_ in (A.OK,) for s_ in statuses),
+            "wall_s_timed_loop": t_wall,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device):
+    import torch
+    from paper_2609_36662_gb300 import aloco as A
+    from paper_2609_36662_gb300 import workloads as W
+    rbytes = w.replica_bytes()
+    h2d = w.numel * (8 + w.M * rbytes)
+    d2h = w.numel * 8
+    try:
+        page = os.sysconf("SC_PAGE_SIZE") * os.sysconf("SC_PHYS_PAGES")
+    except Exception:
+        page = 0
+    if page and (h2d + d2h) > 0.4 * page:
+        return {"value": None, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h,
+                "skipped": "pinned host buffers would exceed 40% of host RAM"}
+    hg = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
+    hv = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
+    hx = [torch.empty(w.numel, dtype=W.replica_dtype(w), pin_memory=True)
+          for _ in range(w.M)]
+    og = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
+    ov = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
+    W.fill_replicas(w, g, xs, 0)
+    hg.copy_(g)
+    hv.copy_(v)
+    for a, b in zip(hx, xs):
+        a.copy_(b)
+    ms = []
+    n_total = args.e2e_warmup + args.e2e_steps
+    for k in range(n_total):
+        step, hsel = rounds[k % len(rounds)]
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            g.copy_(hg, non_blocking=True)
+            v.copy_(hv, non_blocking=True)
+            for a, b in zip(xs, hx):
+                a.copy_(b, non_blocking=True)
+            A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step,
+                   schedule=sched, outer_lr=w.outer_lr,
+                   outer_beta=w.outer_beta, stream=stream)
+            og.copy_(g, non_blocking=True)
+            ov.copy_(v, non_blocking=True)
+            e1.record(stream)
+        e1.synchronize()
+        if k >= args.e2e_warmup:
+            ms.append(e0.elapsed_time(e1))
+    m = reduce_max(statistics.mean(ms), world, device)
+    return {"value": job_value(1.0, m / 1e3, world), "unit": UNIT,
+            "ms_per_step": m, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h + 8 * (w.M + 2),
+            "steps": args.e2e_steps}
+
+
+def main(argv=None):
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
+    p.add_argument("--workload", default=None,
+                   help="workload name (default: the Llama-style 150M set, "
+                        "8 fp32 workers)")
+    p.add_argument("--cpu-seconds", type=float, default=10.0)
+    p.add_argument("--ref-step-seconds", type=float, default=3.0)
+    p.add_argument("--e2e-steps", type=int, default=5)
+    p.add_argument("--e2e-warmup", type=int, default=2)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--list", action="store_true")
+    args = p.parse_args(argv)
+    table = workloads_by_name()
+    if args.list:
+        for name, w in table.items():
+            print(name, w.numel, w.M, w.dtype, w.bytes_per_round())
+        return 0
+    if args.warmup < 3 and args.impl == "cuda":
+        print("warning: fewer than 3 warm-up rounds", file=sys.stderr)
+    name = args.workload or default_workload_name()
+    w = table.get(name) or parse_flat(name)
+    if w is None:
+        p.error(f"unknown workload {name}; --list shows them, or use "
+                "flat<N>_m<M>_<f32|bf16>")
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_cuda(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,228 @@
+/*
+ * aloco.h -- C ABI of libaloco: the AutoLoCo outer synchronisation round
+ * (arxiv 2609.36662) on one GB300 GPU.
+ *
+ * One call runs the whole round of Algorithm 1 ("Synchronization and
+ * corrected outer update" plus the D_t / C_t part of "Interval evaluation")
+ * for M worker replicas that live in the memory of one GPU:
+ *
+ *   Delta_m = theta - x_m                       pseudo-gradients (Alg. 1)
+ *   Dbar    = (1/M) sum_m Delta_m               synchronisation (Alg. 1)
+ *   D       = (1/M) sum_m ||Delta_m||^2         local-drift energy
+ *   C       = M ||Dbar||^2 / (D + eps)          aggregation coherence
+ *                                               (Eq. adaptive-h-core-diagnostics)
+ *   Dtil    = Dbar / (rho + eps)  (optional)    (Eq. normalized-pseudo-gradient,
+ *                                                App. B.3)
+ *   v'      = mu_t v + Dtil
+ *   d       = Dtil + mu_t v'
+ *   theta'  = theta - eta_out d                 (Eq. autoloco-corrected-nesterov)
+ *   x_m     = theta'   for every m              replica reset (Alg. 1)
+ *
+ * with rho, mu_t, kappa_t and eta_out from the Outer Optimizer Correction
+ * (Sec. 3.2; App. B.2 and B.4), evaluated on the host from exact previews of
+ * the inner learning-rate schedule.  The elementwise work is one fused CUDA
+ * pass that reads theta, v and every replica once and writes each once.
+ *
+ * Conventions shared by every entry point:
+ *   - All N-element buffers are caller-owned DEVICE memory on the current
+ *     CUDA device and are updated in place.  `locals` is a HOST array of M
+ *     device pointers.  Buffers must not overlap one another.
+ *   - theta ("global") and v ("momentum") are fp32; replicas are fp32 or
+ *     bf16 (aloco_dtype).  Element n of every buffer is parameter n of the
+ *     flattened parameter vector.
+ *   - Return value: ALOCO_OK (0) or a negative aloco_status.  Arguments are
+ *     validated before any work is enqueued; on ALOCO_ERR_ARG and
+ *     ALOCO_ERR_ALIAS no buffer is touched.  aloco_last_error() returns a
+ *     thread-local message describing the last failure.  The library never
+ *     exits or traps.
+ *   - Work is enqueued on opts->stream (NULL: the legacy default stream).
+ *     aloco_sync / aloco_sync_ex return after the round has completed on
+ *     that stream (they wait for the statistics, a few hundred bytes).
+ *   - Statistics are reduced in a fixed order, so repeated calls on the same
+ *     inputs, device and build return bit-identical results.
+ */
+#ifndef ALOCO_H
+#define ALOCO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ALOCO_MAX_WORKERS 32
+
+/* Replica storage type.  theta and v are always fp32 (the paper keeps FP32
+ * master weights and outer state, App. E.1 and App. G.1). */
+typedef enum { ALOCO_F32 = 0, ALOCO_BF16 = 1 } aloco_dtype;
+
+typedef enum {
+    ALOCO_OK = 0,
+    ALOCO_ERR_ARG = -1,       /* invalid argument; nothing was touched     */
+    ALOCO_ERR_CUDA = -2,      /* a CUDA runtime call failed                */
+    ALOCO_ERR_NONFINITE = -3, /* round completed; some outputs are NaN/Inf */
+    ALOCO_ERR_ALIAS = -4,     /* two buffers overlap; nothing was touched  */
+    ALOCO_ERR_NOMEM = -5      /* workspace allocation failed               */
+} aloco_status;
+
+/* Inner learning-rate schedule (Tab. training settings: cosine decay with a
+ * linear warm-up).  For global inner step s (0-based):
+ *   s <  warmup_steps:            lr = peak_lr * (s + 1) / warmup_steps
+ *   warmup_steps <= s < total:    cosine:  final + (peak - final)(1 + cos(pi f))/2
+ *                                 linear:  peak + (final - peak) f
+ *                                 with f = (s - warmup) / (total - warmup)
+ *   s >= total_steps:             lr = final_lr
+ *   kind CONSTANT:                lr = peak_lr for every s.
+ * total_steps counts the warm-up.  Requirements: 0 <= warmup_steps <
+ * total_steps (any values for CONSTANT), finite non-negative rates. */
+typedef enum {
+    ALOCO_SCHED_COSINE = 0,
+    ALOCO_SCHED_CONSTANT = 1,
+    ALOCO_SCHED_LINEAR = 2
+} aloco_sched_kind;
+
+typedef struct aloco_schedule {
+    int32_t kind; /* aloco_sched_kind */
+    int32_t reserved;
+    double peak_lr;
+    double final_lr;
+    int64_t warmup_steps;
+    int64_t total_steps;
+} aloco_schedule_t;
+
+/* Which parts of the Outer Optimizer Correction run (Tab. component
+ * ablation; App. E.4):
+ *   FULL           mu_t = clip(mu_base^rho, mu_min, mu_max),
+ *                  eta_out = eta_base kappa_t (1 - mu_t)/(1 - mu_base)
+ *   MOMENTUM_ONLY  mu_t as FULL, eta_out = eta_base
+ *   NONE           mu_t = mu_base, eta_out = eta_base (DiLoCo's outer step)
+ * Pseudo-gradient normalisation is switched independently
+ * (aloco_opts_t.normalize; App. B.3). */
+typedef enum {
+    ALOCO_CORR_FULL = 0,
+    ALOCO_CORR_MOMENTUM_ONLY = 1,
+    ALOCO_CORR_NONE = 2
+} aloco_corr_mode;
+
+/* Options.  aloco_default_opts() fills the paper's settings
+ * (Tab. AutoLoCo configuration): mu_min 0.45, mu_max 0.90, kappa_max 1.6,
+ * eps 1e-8, normalize off, FULL correction, no kernel timing, default
+ * stream.  Passing NULL where an opts pointer is accepted means these
+ * defaults. */
+typedef struct aloco_opts {
+    double mu_min;
+    double mu_max;
+    double kappa_max;
+    double eps;           /* the paper's numerical constant epsilon, > 0     */
+    int32_t normalize;    /* 1: Dtil = Dbar / (rho + eps)                    */
+    int32_t mode;         /* aloco_corr_mode                                 */
+    int32_t time_kernel;  /* 1: stats_out->kernel_ms = duration of the fused
+                             pass, from CUDA events on the launch stream     */
+    int32_t reserved;
+    void *stream;         /* cudaStream_t; NULL = legacy default stream      */
+} aloco_opts_t;
+
+/* Correction context of one interval (App. B.2, B.4). */
+typedef struct aloco_correction {
+    double lam_sel;  /* Lambda_t      = sum_{h=1..H_sel}  lr(step + h - 1)   */
+    double lam_base; /* Lambda_t^base = sum_{h=1..H_base} lr(step + h - 1)   */
+    double rho_unc;  /* Lambda_t / (Lambda_t^base + eps)                     */
+    double rho;      /* max(rho_unc, 1)                                      */
+    double mu_t;     /* outer momentum applied this round                    */
+    double kappa_t;  /* bounded outer-step scale                             */
+    double eta_out;  /* outer learning rate applied this round               */
+    double inv_norm; /* 1 / (rho + eps) with normalisation, else 1           */
+} aloco_correction_t;
+
+/* Statistics of one round. */
+typedef struct aloco_stats {
+    double D;                         /* local-drift energy D_t              */
+    double C;                         /* aggregation coherence C_t           */
+    double mean_sq_norm;              /* ||Dbar||_2^2                        */
+    double drift[ALOCO_MAX_WORKERS];  /* ||Delta_m||_2^2, m < M              */
+    aloco_correction_t corr;          /* the correction context applied      */
+    int64_t nonfinite;                /* elements whose theta' or v' is not
+                                         finite                              */
+    int32_t M;
+    int32_t grid;                     /* CUDA blocks of the fused pass       */
+    float kernel_ms;                  /* fused-pass duration, or -1          */
+    int32_t reserved;
+} aloco_stats_t;
+
+/* Fill *opts with the defaults listed above. */
+void aloco_default_opts(aloco_opts_t *opts);
+
+/* Accumulated inner learning rate over an interval of H local steps that
+ * starts at global inner step t0 (0-based):
+ *   sum_{h=1..H} lr(t0 + h - 1)          (Eq. app-outer-correction-lr-masses)
+ * Host-only, no GPU needed.  Returns NaN when schedule is NULL or invalid,
+ * t0 < 0 or H < 0; H = 0 gives 0. */
+double aloco_inner_lr_accum(const aloco_schedule_t *schedule, int64_t t0,
+                            int64_t H);
+
+/* The scalar correction context of an interval starting at global inner
+ * step `step` with selected horizon H_sel and base horizon H_base (both in
+ * executable steps; Sec. 3.2, Eq. outer-correction-ratio,
+ * Eq. adjusted-outer-learning-rate; App. B.2-B.4).  outer_lr is
+ * eta_base^out, outer_beta is mu_base.  Host-only.  Requirements: H_sel >=
+ * 1, H_base >= 1, step >= 0, outer_lr finite, 0 < outer_beta < 1 for FULL
+ * and MOMENTUM_ONLY, 0 <= outer_beta < 1 for NONE, 0 <= mu_min <= mu_max
+ * < 1, kappa_max >= 1, eps > 0. */
+int aloco_correction(const aloco_schedule_t *schedule, int64_t step,
+                     int64_t H_sel, int64_t H_base, double outer_lr,
+                     double outer_beta, const aloco_opts_t *opts,
+                     aloco_correction_t *out);
+
+/* One outer synchronisation round with default options (see
+ * aloco_sync_ex).  Equivalent to aloco_sync_ex(..., NULL). */
+int aloco_sync(float *global, float *momentum, void *const *locals,
+               size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+               int64_t H_base, int64_t step,
+               const aloco_schedule_t *schedule, double outer_lr,
+               double outer_beta, aloco_stats_t *stats_out);
+
+/* One outer synchronisation round (Algorithm 1: synchronisation, corrected
+ * Nesterov outer update, replica reset, D_t and C_t).
+ *   global    [N] fp32 device   theta_t in, theta_{t+1} out
+ *   momentum  [N] fp32 device   v_{t-1} in, v_t out
+ *   locals    host array of M device pointers; locals[m] is [N] of `dtype`,
+ *             worker m's endpoint theta^(m)_{t,H} in, theta_{t+1} out
+ *             (bf16: theta_{t+1} rounded to nearest even)
+ *   N         parameters (0 is allowed: no kernel runs, statistics are 0)
+ *   M         workers, 1 <= M <= ALOCO_MAX_WORKERS
+ *   H_sel, H_base, step   executable horizons and the 0-based global inner
+ *             step at which the interval began (App. B.2)
+ *   schedule  inner learning-rate schedule
+ *   outer_lr, outer_beta  eta_base^out and mu_base
+ *   opts      NULL or options (see aloco_opts_t)
+ *   stats_out NULL or host memory for the statistics
+ * Buffers of any 4-byte (fp32) / 2-byte (bf16) alignment are accepted;
+ * when all of them are 16-byte aligned the fused pass uses 16-byte vector
+ * accesses.  Returns ALOCO_ERR_NONFINITE when some theta' or v' is NaN/Inf
+ * (outputs and statistics are still written; the paper's controller treats
+ * a non-finite statistic as a reduction signal, App. A.2).
+ * Thread safety: calls for the same device are serialised internally. */
+int aloco_sync_ex(float *global, float *momentum, void *const *locals,
+                  size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                  int64_t H_base, int64_t step,
+                  const aloco_schedule_t *schedule, double outer_lr,
+                  double outer_beta, const aloco_opts_t *opts,
+                  aloco_stats_t *stats_out);
+
+/* Message of the last failure on the calling thread ("" if none).  The
+ * pointer stays valid until the next call on this thread. */
+const char *aloco_last_error(void);
+
+/* Release the library's cached per-device workspaces (device and pinned
+ * host memory).  Safe to call at any time no round is in flight. */
+void aloco_shutdown(void);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int aloco_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ALOCO_H */

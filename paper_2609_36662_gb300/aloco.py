@@ -1,0 +1,220 @@
+"""ctypes binding of libaloco (include/aloco.h).
+
+Argument marshalling only: every step of the round runs inside the
+library's CUDA kernels.  If the compiled library is missing this module
+raises on first use; there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional, Sequence
+
+MAX_WORKERS = 32
+
+F32, BF16 = 0, 1
+SCHED_COSINE, SCHED_CONSTANT, SCHED_LINEAR = 0, 1, 2
+CORR_FULL, CORR_MOMENTUM_ONLY, CORR_NONE = 0, 1, 2
+
+OK = 0
+ERR_ARG = -1
+ERR_CUDA = -2
+ERR_NONFINITE = -3
+ERR_ALIAS = -4
+ERR_NOMEM = -5
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
+                         "libaloco.so")
+
+# Names declared in include/aloco.h (checked by the ABI test).
+EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
+           "aloco_sync", "aloco_sync_ex", "aloco_last_error",
+           "aloco_shutdown", "aloco_version")
+
+
+class Schedule(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("peak_lr", ctypes.c_double), ("final_lr", ctypes.c_double),
+                ("warmup_steps", ctypes.c_int64),
+                ("total_steps", ctypes.c_int64)]
+
+    @classmethod
+    def make(cls, kind=SCHED_COSINE, peak_lr=4e-4, final_lr=4e-5,
+             warmup_steps=1000, total_steps=20000):
+        return cls(kind, 0, peak_lr, final_lr, warmup_steps, total_steps)
+
+
+class Opts(ctypes.Structure):
+    _fields_ = [("mu_min", ctypes.c_double), ("mu_max", ctypes.c_double),
+                ("kappa_max", ctypes.c_double), ("eps", ctypes.c_double),
+                ("normalize", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("time_kernel", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("stream", ctypes.c_void_p)]
+
+
+class Correction(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_double) for n in
+                ("lam_sel", "lam_base", "rho_unc", "rho", "mu_t", "kappa_t",
+                 "eta_out", "inv_norm")]
+
+    def as_dict(self):
+        return {n: getattr(self, n) for n, _ in self._fields_}
+
+
+class Stats(ctypes.Structure):
+    _fields_ = [("D", ctypes.c_double), ("C", ctypes.c_double),
+                ("mean_sq_norm", ctypes.c_double),
+                ("drift", ctypes.c_double * MAX_WORKERS),
+                ("corr", Correction), ("nonfinite", ctypes.c_int64),
+                ("M", ctypes.c_int32), ("grid", ctypes.c_int32),
+                ("kernel_ms", ctypes.c_float), ("reserved", ctypes.c_int32)]
+
+    def as_dict(self):
+        return {"D": self.D, "C": self.C, "mean_sq_norm": self.mean_sq_norm,
+                "drift": list(self.drift[:self.M]),
+                "corr": self.corr.as_dict(), "nonfinite": self.nonfinite,
+                "M": self.M, "grid": self.grid, "kernel_ms": self.kernel_ms}
+
+
+class AlocoError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"aloco status {status}: {message}")
+        self.status = status
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def load():
+    """Load libaloco.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(
+            f"{_LIB_PATH} is missing: build it with "
+            "`python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(_LIB_PATH)
+    vp, i64, i32, dbl = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, \
+        ctypes.c_double
+    lib.aloco_default_opts.argtypes = [ctypes.POINTER(Opts)]
+    lib.aloco_default_opts.restype = None
+    lib.aloco_inner_lr_accum.argtypes = [ctypes.POINTER(Schedule), i64, i64]
+    lib.aloco_inner_lr_accum.restype = dbl
+    lib.aloco_correction.argtypes = [ctypes.POINTER(Schedule), i64, i64, i64,
+                                     dbl, dbl, ctypes.POINTER(Opts),
+                                     ctypes.POINTER(Correction)]
+    lib.aloco_correction.restype = i32
+    sync_args = [vp, vp, ctypes.POINTER(vp), ctypes.c_size_t, i32, i32, i64,
+                 i64, i64, ctypes.POINTER(Schedule), dbl, dbl]
+    lib.aloco_sync.argtypes = sync_args + [ctypes.POINTER(Stats)]
+    lib.aloco_sync.restype = i32
+    lib.aloco_sync_ex.argtypes = sync_args + [ctypes.POINTER(Opts),
+                                              ctypes.POINTER(Stats)]
+    lib.aloco_sync_ex.restype = i32
+    lib.aloco_last_error.argtypes = []
+    lib.aloco_last_error.restype = ctypes.c_char_p
+    lib.aloco_shutdown.argtypes = []
+    lib.aloco_shutdown.restype = None
+    lib.aloco_version.argtypes = []
+    lib.aloco_version.restype = i32
+    _lib = lib
+    return lib
+
+
+def last_error() -> str:
+    return load().aloco_last_error().decode()
+
+
+def default_opts(**kw) -> Opts:
+    o = Opts()
+    load().aloco_default_opts(ctypes.byref(o))
+    for k, val in kw.items():
+        setattr(o, k, val)
+    return o
+
+
+def inner_lr_accum(schedule: Schedule, t0: int, H: int) -> float:
+    return load().aloco_inner_lr_accum(ctypes.byref(schedule), t0, H)
+
+
+def correction(schedule: Schedule, step: int, H_sel: int, H_base: int,
+               outer_lr: float, outer_beta: float,
+               opts: Optional[Opts] = None) -> Correction:
+    out = Correction()
+    rc = load().aloco_correction(ctypes.byref(schedule), step, H_sel, H_base,
+                                 outer_lr, outer_beta,
+                                 ctypes.byref(opts) if opts else None,
+                                 ctypes.byref(out))
+    if rc != OK:
+        raise AlocoError(rc, last_error())
+    return out
+
+
+def sync_ptrs(g_ptr: int, v_ptr: int, x_ptrs: Sequence[int], N: int,
+              dtype: int, H_sel: int, H_base: int, step: int,
+              schedule: Schedule, outer_lr: float, outer_beta: float,
+              opts: Optional[Opts] = None, raise_on_error: bool = True):
+    """aloco_sync_ex on raw device addresses.  Returns (status, Stats)."""
+    M = len(x_ptrs)
+    arr = (ctypes.c_void_p * max(M, 1))(*x_ptrs)
+    st = Stats()
+    rc = load().aloco_sync_ex(g_ptr, v_ptr, arr, N, M, dtype, H_sel, H_base,
+                              step, ctypes.byref(schedule), outer_lr,
+                              outer_beta,
+                              ctypes.byref(opts) if opts is not None else None,
+                              ctypes.byref(st))
+    if raise_on_error and rc not in (OK, ERR_NONFINITE):
+        raise AlocoError(rc, last_error())
+    return rc, st
+
+
+def sync(global_, momentum, locals_, *, H_sel: int, H_base: int, step: int,
+         schedule: Schedule, outer_lr: float, outer_beta: float,
+         opts: Optional[Opts] = None, stream=None, raise_on_error=True):
+    """One outer synchronisation round on torch CUDA tensors, in place.
+
+    global_, momentum: contiguous float32 [N]; locals_: M contiguous tensors
+    [N] of float32 or bfloat16.  The round runs on `stream` (default: the
+    current torch stream)."""
+    import torch
+    if global_.dtype != torch.float32 or momentum.dtype != torch.float32:
+        raise TypeError("global and momentum must be float32")
+    N = global_.numel()
+    if momentum.numel() != N or any(x.numel() != N for x in locals_):
+        raise ValueError("all buffers must have the same number of elements")
+    if not locals_:
+        raise ValueError("need at least one replica")
+    rdt = locals_[0].dtype
+    if any(x.dtype != rdt for x in locals_):
+        raise TypeError("replicas must share one dtype")
+    if rdt == torch.float32:
+        dtype = F32
+    elif rdt == torch.bfloat16:
+        dtype = BF16
+    else:
+        raise TypeError(f"unsupported replica dtype {rdt}")
+    for t in (global_, momentum, *locals_):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("buffers must be contiguous CUDA tensors")
+    if opts is None:
+        opts = default_opts()
+    s = stream if stream is not None else torch.cuda.current_stream(
+        global_.device)
+    opts.stream = s.cuda_stream
+    with torch.cuda.device(global_.device):
+        rc, st = sync_ptrs(global_.data_ptr(), momentum.data_ptr(),
+                           [x.data_ptr() for x in locals_], N, dtype, H_sel,
+                           H_base, step, schedule, outer_lr, outer_beta, opts,
+                           raise_on_error)
+    return st.as_dict() | {"status": rc}
+
+
+def shutdown():
+    if _lib is not None:
+        _lib.aloco_shutdown()

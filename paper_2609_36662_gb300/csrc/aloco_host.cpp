@@ -1,0 +1,517 @@
+// Host side of libaloco: argument checks, the scalar Outer Optimizer
+// Correction (Sec. 3.2; App. B.2-B.4), the per-device workspace, the launch
+// of the fused pass and the finalisation of D_t and C_t
+// (Eq. adaptive-h-core-diagnostics).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <memory>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/aloco.h"
+#include "aloco_internal.h"
+
+namespace {
+
+thread_local std::string t_err;
+
+int fail(int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    t_err = buf;
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+    return fail(ALOCO_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorString(e),
+                cudaGetErrorName(e));
+}
+
+// ------------------------------------------------------------- schedule
+
+bool schedule_ok(const aloco_schedule_t *s, std::string *why) {
+    if (!s) { *why = "schedule is NULL"; return false; }
+    if (!(std::isfinite(s->peak_lr) && s->peak_lr >= 0.0)) {
+        *why = "peak_lr must be finite and >= 0"; return false;
+    }
+    if (s->kind == ALOCO_SCHED_CONSTANT) return true;
+    if (s->kind != ALOCO_SCHED_COSINE && s->kind != ALOCO_SCHED_LINEAR) {
+        *why = "unknown schedule kind"; return false;
+    }
+    if (!(std::isfinite(s->final_lr) && s->final_lr >= 0.0)) {
+        *why = "final_lr must be finite and >= 0"; return false;
+    }
+    if (s->warmup_steps < 0 || s->total_steps <= s->warmup_steps) {
+        *why = "need 0 <= warmup_steps < total_steps"; return false;
+    }
+    return true;
+}
+
+// Inner learning rate at global step k (Tab. training settings).
+double lr_at(const aloco_schedule_t &s, int64_t k) {
+    if (s.kind == ALOCO_SCHED_CONSTANT) return s.peak_lr;
+    if (k < s.warmup_steps)
+        return s.peak_lr * (double)(k + 1) / (double)s.warmup_steps;
+    if (k >= s.total_steps) return s.final_lr;
+    const double f = (double)(k - s.warmup_steps) /
+                     (double)(s.total_steps - s.warmup_steps);
+    if (s.kind == ALOCO_SCHED_COSINE)
+        return s.final_lr +
+               0.5 * (s.peak_lr - s.final_lr) * (1.0 + std::cos(M_PI * f));
+    return s.peak_lr + (s.final_lr - s.peak_lr) * f;
+}
+
+// sum_{h=1..H} lr(t0 + h - 1), Neumaier-compensated.  Segments where the
+// rate is constant (constant schedule, the tail after total_steps) are
+// summed as a product.
+double lr_mass(const aloco_schedule_t &s, int64_t t0, int64_t H) {
+    if (H <= 0) return 0.0;
+    if (s.kind == ALOCO_SCHED_CONSTANT) return (double)H * s.peak_lr;
+    const int64_t end = t0 + H;  // exclusive
+    const int64_t vary_end = end < s.total_steps ? end : s.total_steps;
+    double sum = 0.0, comp = 0.0;
+    for (int64_t k = t0; k < vary_end; ++k) {
+        const double x = lr_at(s, k);
+        const double t = sum + x;
+        comp += std::fabs(sum) >= std::fabs(x) ? (sum - t) + x : (x - t) + sum;
+        sum = t;
+    }
+    const int64_t tail_begin = t0 > s.total_steps ? t0 : s.total_steps;
+    if (end > tail_begin) {
+        const double x = (double)(end - tail_begin) * s.final_lr;
+        const double t = sum + x;
+        comp += std::fabs(sum) >= std::fabs(x) ? (sum - t) + x : (x - t) + sum;
+        sum = t;
+    }
+    return sum + comp;
+}
+
+// ----------------------------------------------------------- correction
+
+int correction_impl(const aloco_schedule_t *sched, int64_t step,
+                    int64_t H_sel, int64_t H_base, double outer_lr,
+                    double outer_beta, const aloco_opts_t &o,
+                    aloco_correction_t *out) {
+    std::string why;
+    if (!schedule_ok(sched, &why)) return fail(ALOCO_ERR_ARG, "%s", why.c_str());
+    if (H_sel < 1 || H_base < 1)
+        return fail(ALOCO_ERR_ARG, "H_sel (%lld) and H_base (%lld) must be >= 1",
+                    (long long)H_sel, (long long)H_base);
+    if (step < 0) return fail(ALOCO_ERR_ARG, "step must be >= 0");
+    if (!std::isfinite(outer_lr)) return fail(ALOCO_ERR_ARG, "outer_lr must be finite");
+    if (o.mode != ALOCO_CORR_FULL && o.mode != ALOCO_CORR_MOMENTUM_ONLY &&
+        o.mode != ALOCO_CORR_NONE)
+        return fail(ALOCO_ERR_ARG, "unknown correction mode %d", o.mode);
+    const bool beta_ok = o.mode == ALOCO_CORR_NONE
+                             ? (outer_beta >= 0.0 && outer_beta < 1.0)
+                             : (outer_beta > 0.0 && outer_beta < 1.0);
+    if (!beta_ok)
+        return fail(ALOCO_ERR_ARG, "outer_beta %g out of range for mode %d",
+                    outer_beta, o.mode);
+    if (!(o.eps > 0.0 && std::isfinite(o.eps)))
+        return fail(ALOCO_ERR_ARG, "eps must be finite and > 0");
+    if (!(o.mu_min >= 0.0 && o.mu_min <= o.mu_max && o.mu_max < 1.0))
+        return fail(ALOCO_ERR_ARG, "need 0 <= mu_min <= mu_max < 1");
+    if (!(o.kappa_max >= 1.0 && std::isfinite(o.kappa_max)))
+        return fail(ALOCO_ERR_ARG, "kappa_max must be finite and >= 1");
+
+    aloco_correction_t c;
+    // Eq. app-outer-correction-lr-masses: both previews start at s_t = step.
+    c.lam_sel = lr_mass(*sched, step, H_sel);
+    c.lam_base = lr_mass(*sched, step, H_base);
+    // Eq. app-outer-correction-ratios.
+    c.rho_unc = c.lam_sel / (c.lam_base + o.eps);
+    c.rho = std::fmax(c.rho_unc, 1.0);
+    if (o.mode == ALOCO_CORR_NONE) {
+        c.mu_t = outer_beta;
+        c.kappa_t = 1.0;
+        c.eta_out = outer_lr;
+    } else {
+        // Momentum retention mu_base^rho, clipped (Sec. 3.2; App. B.4).
+        c.mu_t = std::fmin(std::fmax(std::pow(outer_beta, c.rho), o.mu_min),
+                           o.mu_max);
+        if (o.mode == ALOCO_CORR_MOMENTUM_ONLY) {
+            c.kappa_t = 1.0;
+            c.eta_out = outer_lr;
+        } else {
+            // Eq. app-outer-step-scale, Eq. app-adjusted-outer-learning-rate.
+            c.kappa_t = std::fmin(c.rho, o.kappa_max);
+            c.eta_out = outer_lr * c.kappa_t * (1.0 - c.mu_t) / (1.0 - outer_beta);
+        }
+    }
+    // Eq. normalized-pseudo-gradient with rho + eps (App. B.3).
+    c.inv_norm = o.normalize ? 1.0 / (c.rho + o.eps) : 1.0;
+    *out = c;
+    return ALOCO_OK;
+}
+
+// ------------------------------------------------------------ workspace
+
+// Layout of the device workspace of one device (one allocation).
+struct Workspace {
+    std::mutex mu;
+    bool ready = false;
+    int device = -1;
+    int sm_count = 0;
+    int max_grid = 0;
+    char *dev = nullptr;                  // device block
+    double *partials = nullptr;           // [max_grid * (MAX_WORKERS + 1)]
+    unsigned long long *nf_partials = nullptr;  // [max_grid]
+    double *totals = nullptr;             // [MAX_WORKERS + 1] then nf_total
+    unsigned long long *nf_total = nullptr;
+    unsigned int *ticket = nullptr;
+    double *host = nullptr;               // pinned readback of totals + nf
+    cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+};
+
+constexpr int kTotals = ALOCO_MAX_WORKERS + 2;  // totals + nf slot (8 B each)
+
+std::mutex g_registry_mu;
+std::vector<std::unique_ptr<Workspace>> g_registry;
+
+Workspace *workspace_for(int device) {
+    std::lock_guard<std::mutex> lk(g_registry_mu);
+    if ((int)g_registry.size() <= device) g_registry.resize(device + 1);
+    if (!g_registry[device]) g_registry[device].reset(new Workspace());
+    return g_registry[device].get();
+}
+
+// Allocate on first use (caller holds ws->mu, device is current).
+int ensure_ready(Workspace *ws, int device) {
+    if (ws->ready) return ALOCO_OK;
+    cudaError_t e = cudaDeviceGetAttribute(&ws->sm_count,
+                                           cudaDevAttrMultiProcessorCount, device);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    int max_threads = 0;
+    e = cudaDeviceGetAttribute(&max_threads,
+                               cudaDevAttrMaxThreadsPerMultiProcessor, device);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    ws->max_grid = ws->sm_count * (max_threads / aloco::kBlock);
+    const size_t n_part = (size_t)ws->max_grid * (ALOCO_MAX_WORKERS + 1);
+    const size_t bytes = n_part * sizeof(double) +
+                         (size_t)ws->max_grid * sizeof(unsigned long long) +
+                         kTotals * sizeof(double) + 256;
+    e = cudaMalloc((void **)&ws->dev, bytes);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(ALOCO_ERR_NOMEM, "workspace cudaMalloc(%zu): %s", bytes,
+                    cudaGetErrorString(e));
+    }
+    char *p = ws->dev;
+    ws->partials = (double *)p;
+    p += n_part * sizeof(double);
+    ws->nf_partials = (unsigned long long *)p;
+    p += (size_t)ws->max_grid * sizeof(unsigned long long);
+    ws->totals = (double *)p;
+    ws->nf_total = (unsigned long long *)(ws->totals + ALOCO_MAX_WORKERS + 1);
+    p += kTotals * sizeof(double);
+    ws->ticket = (unsigned int *)p;
+    e = cudaMemset(ws->dev, 0, bytes);
+    if (e == cudaSuccess) e = cudaMallocHost((void **)&ws->host, kTotals * sizeof(double));
+    if (e == cudaSuccess) e = cudaEventCreate(&ws->ev0);
+    if (e == cudaSuccess) e = cudaEventCreate(&ws->ev1);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return cuda_fail(e, "workspace setup");
+    }
+    ws->device = device;
+    ws->ready = true;
+    return ALOCO_OK;
+}
+
+// --------------------------------------------------------- buffer checks
+
+typedef CUresult (*GetAddressRangeFn)(CUdeviceptr *, size_t *, CUdeviceptr);
+
+GetAddressRangeFn address_range_fn() {
+    static GetAddressRangeFn fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &p, 12000,
+                                             cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            return (GetAddressRangeFn) nullptr;
+        }
+        return (GetAddressRangeFn)p;
+    }();
+    return fn;
+}
+
+// The buffer must be device (or managed) memory of `device`, and when the
+// driver can tell, [p, p + bytes) must lie inside one allocation.
+int check_buffer(const void *p, size_t bytes, int device, const char *name) {
+    cudaPointerAttributes at;
+    cudaError_t e = cudaPointerGetAttributes(&at, p);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(ALOCO_ERR_ARG, "%s: not a CUDA pointer (%s)", name,
+                    cudaGetErrorString(e));
+    }
+    if (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged)
+        return fail(ALOCO_ERR_ARG, "%s: not device memory", name);
+    if (at.type == cudaMemoryTypeDevice && at.device != device)
+        return fail(ALOCO_ERR_ARG, "%s: lives on device %d, current device is %d",
+                    name, at.device, device);
+    if (GetAddressRangeFn fn = address_range_fn()) {
+        CUdeviceptr base = 0;
+        size_t size = 0;
+        if (fn(&base, &size, (CUdeviceptr)p) == CUDA_SUCCESS && size > 0) {
+            if ((uintptr_t)p + bytes > (uintptr_t)base + size)
+                return fail(ALOCO_ERR_ARG,
+                            "%s: %zu bytes from %p run past the end of its "
+                            "allocation (%zu bytes at %p)",
+                            name, bytes, p, size, (void *)base);
+        }
+    }
+    return ALOCO_OK;
+}
+
+void fill_default_opts(aloco_opts_t *o) {
+    std::memset(o, 0, sizeof *o);
+    o->mu_min = 0.45;
+    o->mu_max = 0.90;
+    o->kappa_max = 1.6;
+    o->eps = 1e-8;
+    o->normalize = 0;
+    o->mode = ALOCO_CORR_FULL;
+    o->time_kernel = 0;
+    o->stream = nullptr;
+}
+
+// x ~= hi + lo with hi = fl32(x), lo = fl32(x - hi).
+void split_coef(double x, float *hi, float *lo) {
+    *hi = (float)x;
+    *lo = (float)(x - (double)*hi);
+}
+
+void finalize_stats(const double *totals, unsigned long long nf, int M,
+                    double eps, aloco_stats_t *st) {
+    double sum = 0.0;
+    for (int m = 0; m < M; ++m) {
+        st->drift[m] = totals[m];
+        sum += totals[m];
+    }
+    st->D = sum / (double)M;
+    // The pass accumulates S^2 with S = sum_m Delta_m = M * Dbar.
+    st->mean_sq_norm = totals[M] / ((double)M * (double)M);
+    st->C = (double)M * st->mean_sq_norm / (st->D + eps);
+    st->nonfinite = (int64_t)nf;
+}
+
+}  // namespace
+
+// ================================================================ C ABI
+
+extern "C" {
+
+void aloco_default_opts(aloco_opts_t *opts) {
+    if (opts) fill_default_opts(opts);
+}
+
+double aloco_inner_lr_accum(const aloco_schedule_t *schedule, int64_t t0,
+                            int64_t H) {
+    std::string why;
+    if (!schedule_ok(schedule, &why) || t0 < 0 || H < 0) {
+        fail(ALOCO_ERR_ARG, "aloco_inner_lr_accum: %s",
+             why.empty() ? "t0 and H must be >= 0" : why.c_str());
+        return std::nan("");
+    }
+    return lr_mass(*schedule, t0, H);
+}
+
+int aloco_correction(const aloco_schedule_t *schedule, int64_t step,
+                     int64_t H_sel, int64_t H_base, double outer_lr,
+                     double outer_beta, const aloco_opts_t *opts,
+                     aloco_correction_t *out) {
+    aloco_opts_t o;
+    if (opts) o = *opts; else fill_default_opts(&o);
+    if (!out) return fail(ALOCO_ERR_ARG, "out is NULL");
+    return correction_impl(schedule, step, H_sel, H_base, outer_lr, outer_beta,
+                           o, out);
+}
+
+int aloco_sync(float *global, float *momentum, void *const *locals, size_t N,
+               int M, aloco_dtype dtype, int64_t H_sel, int64_t H_base,
+               int64_t step, const aloco_schedule_t *schedule, double outer_lr,
+               double outer_beta, aloco_stats_t *stats_out) {
+    return aloco_sync_ex(global, momentum, locals, N, M, dtype, H_sel, H_base,
+                         step, schedule, outer_lr, outer_beta, nullptr,
+                         stats_out);
+}
+
+int aloco_sync_ex(float *global, float *momentum, void *const *locals,
+                  size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                  int64_t H_base, int64_t step,
+                  const aloco_schedule_t *schedule, double outer_lr,
+                  double outer_beta, const aloco_opts_t *opts,
+                  aloco_stats_t *stats_out) {
+    aloco_opts_t o;
+    if (opts) o = *opts; else fill_default_opts(&o);
+    aloco_stats_t local_stats;
+    aloco_stats_t *st = stats_out ? stats_out : &local_stats;
+
+    // ---------------------------------------------------- arguments
+    if (M < 1 || M > ALOCO_MAX_WORKERS)
+        return fail(ALOCO_ERR_ARG, "M = %d outside [1, %d]", M, ALOCO_MAX_WORKERS);
+    if (dtype != ALOCO_F32 && dtype != ALOCO_BF16)
+        return fail(ALOCO_ERR_ARG, "unknown replica dtype %d", (int)dtype);
+    if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
+    if (N > 0 && (!global || !momentum || !locals))
+        return fail(ALOCO_ERR_ARG, "NULL buffer");
+    for (int m = 0; N > 0 && m < M; ++m)
+        if (!locals[m]) return fail(ALOCO_ERR_ARG, "locals[%d] is NULL", m);
+    aloco_correction_t corr;
+    int rc = correction_impl(schedule, step, H_sel, H_base, outer_lr,
+                             outer_beta, o, &corr);
+    if (rc != ALOCO_OK) return rc;
+
+    std::memset(st, 0, sizeof *st);
+    st->corr = corr;
+    st->M = M;
+    st->kernel_ms = -1.f;
+    if (N == 0) {
+        t_err.clear();
+        return ALOCO_OK;
+    }
+
+    const size_t rsz = dtype == ALOCO_F32 ? 4 : 2;
+    // Pairwise overlap check of the M + 2 byte ranges.
+    {
+        std::vector<std::pair<uintptr_t, size_t>> r;
+        r.push_back({(uintptr_t)global, N * 4});
+        r.push_back({(uintptr_t)momentum, N * 4});
+        for (int m = 0; m < M; ++m) r.push_back({(uintptr_t)locals[m], N * rsz});
+        for (size_t i = 0; i < r.size(); ++i)
+            for (size_t j = i + 1; j < r.size(); ++j)
+                if (r[i].first < r[j].first + r[j].second &&
+                    r[j].first < r[i].first + r[i].second)
+                    return fail(ALOCO_ERR_ALIAS, "buffers %zu and %zu overlap", i, j);
+    }
+    if (((uintptr_t)global | (uintptr_t)momentum) & 3)
+        return fail(ALOCO_ERR_ARG, "global/momentum not 4-byte aligned");
+    for (int m = 0; m < M; ++m)
+        if ((uintptr_t)locals[m] & (rsz - 1))
+            return fail(ALOCO_ERR_ARG, "locals[%d] not %zu-byte aligned", m, rsz);
+
+    int device = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    Workspace *ws = workspace_for(device);
+    std::lock_guard<std::mutex> lk(ws->mu);
+    rc = ensure_ready(ws, device);
+    if (rc != ALOCO_OK) return rc;
+
+    if ((rc = check_buffer(global, N * 4, device, "global")) != ALOCO_OK) return rc;
+    if ((rc = check_buffer(momentum, N * 4, device, "momentum")) != ALOCO_OK) return rc;
+    for (int m = 0; m < M; ++m) {
+        char name[32];
+        snprintf(name, sizeof name, "locals[%d]", m);
+        if ((rc = check_buffer(locals[m], N * rsz, device, name)) != ALOCO_OK)
+            return rc;
+    }
+
+    // ------------------------------------------------------- launch
+    aloco::SyncArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.g = global;
+    a.v = momentum;
+    uintptr_t align_or = (uintptr_t)global | (uintptr_t)momentum;
+    for (int m = 0; m < M; ++m) {
+        a.x[m] = locals[m];
+        align_or |= (uintptr_t)locals[m];
+    }
+    const int pack = aloco::pack_elems(dtype);
+    a.n = (int64_t)N;
+    a.nvec = (align_or & 15) == 0 ? (int64_t)(N / pack) : 0;
+    split_coef(corr.inv_norm / (double)M, &a.c_hi, &a.c_lo);
+    split_coef(corr.mu_t, &a.mu_hi, &a.mu_lo);
+    split_coef(-corr.eta_out, &a.neg_eta_hi, &a.neg_eta_lo);
+    a.M = M;
+    a.partials = ws->partials;
+    a.nf_partials = ws->nf_partials;
+    a.ticket = ws->ticket;
+    a.totals = ws->totals;
+    a.nf_total = ws->nf_total;
+
+    const int64_t work = a.nvec > 0 ? a.nvec : a.n;
+    aloco::LaunchPlan plan;
+    e = dtype == ALOCO_F32 ? aloco::plan_sync_f32(M, work, ws->sm_count, &plan)
+                           : aloco::plan_sync_bf16(M, work, ws->sm_count, &plan);
+    if (e != cudaSuccess) return cuda_fail(e, "launch plan");
+    if (plan.grid > ws->max_grid)
+        return fail(ALOCO_ERR_CUDA, "grid %d exceeds workspace %d", plan.grid,
+                    ws->max_grid);
+
+    cudaStream_t stream = (cudaStream_t)o.stream;
+    if (o.time_kernel && (e = cudaEventRecord(ws->ev0, stream)) != cudaSuccess)
+        return cuda_fail(e, "cudaEventRecord");
+    void *params[] = {&a};
+    e = cudaLaunchKernel(plan.kernel, dim3(plan.grid), dim3(plan.block), params,
+                         0, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "fused sync launch");
+    if (o.time_kernel && (e = cudaEventRecord(ws->ev1, stream)) != cudaSuccess)
+        return cuda_fail(e, "cudaEventRecord");
+    e = cudaMemcpyAsync(ws->host, ws->totals, kTotals * sizeof(double),
+                        cudaMemcpyDeviceToHost, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "statistics readback");
+    e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return cuda_fail(e, "round");
+
+    unsigned long long nf;
+    std::memcpy(&nf, ws->host + ALOCO_MAX_WORKERS + 1, sizeof nf);
+    finalize_stats(ws->host, nf, M, o.eps, st);
+    st->grid = plan.grid;
+    if (o.time_kernel) {
+        float ms = -1.f;
+        if (cudaEventElapsedTime(&ms, ws->ev0, ws->ev1) == cudaSuccess)
+            st->kernel_ms = ms;
+        else
+            cudaGetLastError();
+    }
+    if (st->nonfinite > 0 || !std::isfinite(st->D) || !std::isfinite(st->C))
+        return fail(ALOCO_ERR_NONFINITE,
+                    "round produced %lld non-finite elements (D=%g, C=%g)",
+                    (long long)st->nonfinite, st->D, st->C);
+    t_err.clear();
+    return ALOCO_OK;
+}
+
+const char *aloco_last_error(void) { return t_err.c_str(); }
+
+void aloco_shutdown(void) {
+    std::lock_guard<std::mutex> lk(g_registry_mu);
+    int prev = -1;
+    cudaGetDevice(&prev);
+    for (auto &ws : g_registry) {
+        if (!ws) continue;
+        std::lock_guard<std::mutex> lk2(ws->mu);
+        if (!ws->ready) continue;
+        cudaSetDevice(ws->device);
+        cudaDeviceSynchronize();
+        if (ws->ev0) cudaEventDestroy(ws->ev0);
+        if (ws->ev1) cudaEventDestroy(ws->ev1);
+        if (ws->host) cudaFreeHost(ws->host);
+        if (ws->dev) cudaFree(ws->dev);
+        ws->ev0 = ws->ev1 = nullptr;
+        ws->host = nullptr;
+        ws->dev = nullptr;
+        ws->ready = false;
+    }
+    if (prev >= 0) cudaSetDevice(prev);
+    cudaGetLastError();
+}
+
+int aloco_version(void) { return 100; }
+
+}  // extern "C"

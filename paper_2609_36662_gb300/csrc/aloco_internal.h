@@ -1,0 +1,55 @@
+// Internal interface between the host side of libaloco (aloco_host.cpp) and
+// the fused synchronisation kernels (aloco_sync_*.cu).  Not part of the ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/aloco.h"
+
+namespace aloco {
+
+// Threads per block of the fused pass.
+constexpr int kBlock = 256;
+
+// Everything the fused pass needs, passed by value as a __grid_constant__
+// kernel parameter (the replica pointers are uniform across the grid).
+struct SyncArgs {
+    float *g;                       // theta [n]
+    float *v;                       // momentum [n]
+    void *x[ALOCO_MAX_WORKERS];     // replicas [n] each
+    int64_t n;                      // elements
+    int64_t nvec;                   // packs handled by the vector loop
+                                    // (0 when a buffer is not 16 B aligned)
+    // Round coefficients, each as an fp32 pair hi + lo whose sum carries the
+    // fp64 host value to ~2^-48 relative, so that the per-element update is
+    // not biased by one fixed fp32 rounding of the coefficient.
+    float c_hi, c_lo;               // inv_norm / M  (Dtil = c * sum_m Delta_m)
+    float mu_hi, mu_lo;             // mu_t
+    float neg_eta_hi, neg_eta_lo;   // -eta_out
+    int M;
+    // workspace (device)
+    double *partials;               // [grid][M + 1]: sum Delta_m^2 (m < M), sum S^2
+    unsigned long long *nf_partials;// [grid]
+    unsigned int *ticket;           // last-block-done counter, 0 between launches
+    double *totals;                 // [M + 1] fixed-order totals
+    unsigned long long *nf_total;   // [1]
+};
+
+// Elements per vector pack: one 16-byte access of a replica.
+inline int pack_elems(aloco_dtype dt) { return dt == ALOCO_F32 ? 4 : 8; }
+
+// Launch configuration chosen for (M, dtype, n) on the current device.
+struct LaunchPlan {
+    const void *kernel;
+    int grid;
+    int block;
+};
+
+// Pick the kernel instance and grid; returns cudaSuccess or an error.
+cudaError_t plan_sync_f32(int M, int64_t work_items, int sm_count,
+                          LaunchPlan *plan);
+cudaError_t plan_sync_bf16(int M, int64_t work_items, int sm_count,
+                           LaunchPlan *plan);
+
+}  // namespace aloco

@@ -1,0 +1,9 @@
+// bf16-replica instances of the fused synchronisation pass.
+#include "aloco_sync_kernel.cuh"
+
+namespace aloco {
+cudaError_t plan_sync_bf16(int M, int64_t work_items, int sm_count,
+                           LaunchPlan *plan) {
+    return plan_dispatch<true>(M, work_items, sm_count, plan);
+}
+}  // namespace aloco

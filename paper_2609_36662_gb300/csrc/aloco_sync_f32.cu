@@ -1,0 +1,9 @@
+// fp32-replica instances of the fused synchronisation pass.
+#include "aloco_sync_kernel.cuh"
+
+namespace aloco {
+cudaError_t plan_sync_f32(int M, int64_t work_items, int sm_count,
+                          LaunchPlan *plan) {
+    return plan_dispatch<false>(M, work_items, sm_count, plan);
+}
+}  // namespace aloco

@@ -186,17 +186,30 @@ def _segments(w: Workload):
     return segs
 
 
-CHUNK = 1 << 26   # elements drawn per generator call (bounds scratch memory)
+CHUNK = 1 << 24   # elements per generator chunk (bounds scratch memory)
 
 
-def make_global(w: Workload, device="cpu", seed_offset: int = 0):
-    """theta_global ~ N(0, 0.02) (fp32); norm vectors set to 1.0."""
-    gen = torch.Generator(device=device).manual_seed(
-        1_000_003 * w.seed + seed_offset)
+def _chunk_gen(device, *key):
+    """A generator whose seed depends only on `key`, so any chunk of any
+    round can be drawn on its own."""
+    seed = 0
+    for k in key:
+        seed = (seed * 1_000_003 + int(k) + 17) % (1 << 62)
+    return torch.Generator(device=device).manual_seed(seed)
+
+
+def n_chunks(w: Workload) -> int:
+    return (w.numel + CHUNK - 1) // CHUNK
+
+
+def make_global(w: Workload, device="cpu", draw: int = 0):
+    """theta_global ~ N(0, 0.02) (fp32); norm vectors set to 1.0.  `draw`
+    selects an independent draw of the same distribution."""
     g = torch.empty(w.numel, dtype=torch.float32, device=device)
-    for s in range(0, w.numel, CHUNK):
-        e = min(w.numel, s + CHUNK)
-        g[s:e].normal_(0.0, 0.02, generator=gen)
+    key = 0 if draw == 0 else 10_000 + draw
+    for c in range(n_chunks(w)):
+        s, e = c * CHUNK, min(w.numel, (c + 1) * CHUNK)
+        g[s:e].normal_(0.0, 0.02, generator=_chunk_gen(device, w.seed, key, c))
     if w.shape is not None:
         for off, n, _, is_norm in _segments(w):
             if is_norm:
@@ -217,26 +230,39 @@ def alloc_replicas(w: Workload, device="cpu"):
     return [torch.empty(w.numel, dtype=dt, device=device) for _ in range(w.M)]
 
 
-def fill_replicas(w: Workload, g: torch.Tensor, replicas, round_index: int):
-    """Write x_m = g + sigma_l (a s + b e_m) into the given replica buffers
-    (computed in fp32, then stored in the replica dtype, round to nearest
-    even for bf16).  Deterministic in (w.seed, round_index)."""
-    device = g.device
-    gen = torch.Generator(device=device).manual_seed(
-        7919 * w.seed + 104_729 * (round_index + 1))
-    segs = _segments(w)
-    for s in range(0, w.numel, CHUNK):
-        e = min(w.numel, s + CHUNK)
-        n = e - s
-        sigma = _sigma_slice(segs, s, e, device)
-        shared = torch.randn(n, generator=gen, device=device,
-                             dtype=torch.float32)
-        shared.mul_(w.noise_a)
-        for x in replicas:
-            priv = torch.randn(n, generator=gen, device=device,
-                               dtype=torch.float32)
-            priv.mul_(w.noise_b).add_(shared).mul_(sigma).add_(g[s:e])
-            x[s:e].copy_(priv)
+def replica_chunk(w: Workload, g_chunk: torch.Tensor, round_index: int,
+                  c: int):
+    """The M endpoints of chunk c (elements [c*CHUNK, ...)) for round
+    `round_index`, as fp32: x_m = g + sigma_l (a s + b e_m)."""
+    device = g_chunk.device
+    s = c * CHUNK
+    n = g_chunk.numel()
+    gen = _chunk_gen(device, w.seed, round_index + 1, c)
+    sigma = _sigma_slice(_segments(w), s, s + n, device)
+    shared = torch.randn(n, generator=gen, device=device, dtype=torch.float32)
+    shared.mul_(w.noise_a)
+    out = []
+    for _ in range(w.M):
+        priv = torch.randn(n, generator=gen, device=device,
+                           dtype=torch.float32)
+        priv.mul_(w.noise_b).add_(shared).mul_(sigma).add_(g_chunk)
+        out.append(priv)
+    return out
+
+
+def fill_replicas(w: Workload, g: torch.Tensor, replicas, round_index: int,
+                  c_lo: int = 0, c_hi: Optional[int] = None):
+    """Write the endpoints of chunks [c_lo, c_hi) of round `round_index` into
+    the replica buffers (stored in the replica dtype; bf16 by round to
+    nearest even).  `g` and the buffers cover the same element range, which
+    starts at chunk c_lo."""
+    c_hi = n_chunks(w) if c_hi is None else c_hi
+    base = c_lo * CHUNK
+    for c in range(c_lo, c_hi):
+        s, e = c * CHUNK, min(w.numel, (c + 1) * CHUNK)
+        xs = replica_chunk(w, g[s - base:e - base], round_index, c)
+        for x, r in zip(xs, replicas):
+            r[s - base:e - base].copy_(x)
     return replicas
 
 

@@ -1,0 +1,368 @@
+"""Helpers shared by the parity tests: run the CUDA path and the oracle on the
+same seeded inputs and compare them.
+
+Tolerances (written here, used by every parity test):
+  * theta' and v' (fp32 on the GPU, fp64 in the oracle):
+        |gpu - oracle| <= 1e-5 * max(|oracle|, rms(oracle field))
+  * fp32 replicas: the same bound (they hold theta');
+  * bf16 replicas: |gpu - oracle| <= 1 bf16 ulp (at the oracle's value)
+    plus theta's own field tolerance.  The GPU rounds its fp32 theta' to
+    bf16, the oracle its fp64 theta': the two roundings can differ by one
+    step, and by more only where theta' itself differs by more than a bf16
+    step, which happens where theta - eta d cancels to a value far below the
+    field's scale.  In addition, every GPU bf16 replica must be exactly the
+    round-to-nearest-even of the GPU's own theta' (a property, not a
+    comparison with the oracle);
+  * D, C, ||Dbar||^2 and each ||Delta_m||^2: relative 1e-6;
+  * correction scalars (both fp64, on the host): relative 1e-12;
+  * integer outputs (non-finite count): exact.
+"""
+from __future__ import annotations
+
+import concurrent.futures as cf
+
+import numpy as np
+import torch
+
+import oracle as O
+from paper_2609_36662_gb300 import aloco as A
+from paper_2609_36662_gb300 import workloads as W
+
+RTOL_FIELD = 1e-5
+RTOL_STAT = 1e-6
+RTOL_SCALAR = 1e-12
+
+
+def to_numpy_bits(x: torch.Tensor) -> np.ndarray:
+    """Host copy of a replica: float32 values or bf16 bit patterns."""
+    if x.dtype == torch.bfloat16:
+        return x.detach().cpu().view(torch.int16).numpy().view(np.uint16)
+    return x.detach().cpu().numpy()
+
+
+def oracle_dtype(t: torch.dtype) -> int:
+    return O.F32 if t == torch.float32 else O.BF16
+
+
+def schedule_pair(spec: W.ScheduleSpec):
+    return (A.Schedule.make(spec.kind, spec.peak_lr, spec.final_lr,
+                            spec.warmup_steps, spec.total_steps),
+            O.Schedule(spec.kind, spec.peak_lr, spec.final_lr,
+                       spec.warmup_steps, spec.total_steps))
+
+
+def field_error(gpu: np.ndarray, orc: np.ndarray) -> float:
+    gpu = np.asarray(gpu, np.float64)
+    orc = np.asarray(orc, np.float64)
+    if orc.size == 0:
+        return 0.0
+    rms = float(np.sqrt(np.mean(orc * orc)))
+    scale = np.maximum(np.abs(orc), max(rms, 1e-300))
+    err = np.abs(gpu - orc) / scale
+    err[(gpu == orc)] = 0.0
+    return float(err.max())
+
+
+def assert_field(gpu, orc, name, rtol=RTOL_FIELD):
+    e = field_error(gpu, orc)
+    assert e <= rtol, f"{name}: max scaled error {e:.3e} > {rtol:.0e}"
+
+
+def fp32_ulp(values) -> np.ndarray:
+    """Spacing of fp32 numbers at |values|."""
+    a = np.abs(np.asarray(values, np.float64))
+    e = np.floor(np.log2(np.maximum(a, 2.0 ** -126)))
+    return np.exp2(np.maximum(e, -126) - 23)
+
+
+def assert_field_after_chain(gpu, orc, theta_orc, rounds, name,
+                             rtol=RTOL_FIELD):
+    """Final state of two independent multi-round chains.  Each chain stores
+    theta in fp32 between rounds; where the two roundings of theta differ
+    (one fp32 step), the next round's pseudo-gradients differ by that step,
+    and the state carries it on with gain at most one per round.  So on top
+    of the per-round field tolerance each element may differ by up to
+    `rounds` fp32 steps of its theta; the whole-vector relative L2 error
+    must still be within the field tolerance."""
+    gpu = np.asarray(gpu, np.float64)
+    orc = np.asarray(orc, np.float64)
+    rms = float(np.sqrt(np.mean(orc * orc)))
+    tol = rtol * np.maximum(np.abs(orc), rms) + rounds * fp32_ulp(theta_orc)
+    bad = np.abs(gpu - orc) > tol
+    assert not bad.any(), (f"{name}: {int(bad.sum())} elements beyond the "
+                           f"chain tolerance, e.g. index {int(np.argmax(bad))}")
+    l2 = float(np.linalg.norm(gpu - orc) / max(np.linalg.norm(orc), 1e-300))
+    assert l2 <= rtol, f"{name}: relative L2 error {l2:.3e}"
+
+
+def bf16_order_key(bits: np.ndarray) -> np.ndarray:
+    b = bits.astype(np.int64)
+    return np.where(b & 0x8000, -(b & 0x7FFF), b)
+
+
+def bf16_ulp(values: np.ndarray) -> np.ndarray:
+    """Spacing of bf16 numbers at |values| (8 significant bits)."""
+    a = np.abs(np.asarray(values, np.float64))
+    e = np.floor(np.log2(np.maximum(a, 2.0 ** -126)))
+    return np.exp2(np.maximum(e, -126) - 7)
+
+
+def assert_bf16_replica(gpu_bits, orc_bits, orc_theta, name,
+                        rtol=RTOL_FIELD, extra_abs=0.0):
+    gv = O.bf16_bits_to_float(gpu_bits)
+    ov = O.bf16_bits_to_float(orc_bits)
+    orc_theta = np.asarray(orc_theta, np.float64)
+    rms = float(np.sqrt(np.mean(orc_theta * orc_theta))) if orc_theta.size \
+        else 0.0
+    tol = bf16_ulp(ov) + rtol * np.maximum(np.abs(orc_theta), rms) + extra_abs
+    bad = np.abs(gv - ov) > tol
+    assert not bad.any(), (f"{name}: {int(bad.sum())} bf16 replicas beyond one "
+                           f"ulp + field tolerance, e.g. index "
+                           f"{int(np.argmax(bad))}")
+
+
+def assert_bf16_is_rounded_theta(gpu_bits, gpu_theta: torch.Tensor, name):
+    want = gpu_theta.detach().cpu().to(torch.bfloat16).view(torch.int16) \
+        .numpy().view(np.uint16)
+    assert np.array_equal(gpu_bits, want), \
+        f"{name} is not the bf16 rounding of theta'"
+
+
+def assert_rel(gpu, orc, name, rtol):
+    if orc == 0.0:
+        assert gpu == 0.0 or abs(gpu) < 1e-300, f"{name}: {gpu} vs 0"
+        return
+    r = abs(gpu - orc) / abs(orc)
+    assert r <= rtol, f"{name}: {gpu!r} vs {orc!r} (rel {r:.3e} > {rtol:.0e})"
+
+
+def assert_stats(st: dict, orc: dict, M: int):
+    assert_rel(st["D"], orc["D"], "D", RTOL_STAT)
+    assert_rel(st["C"], orc["C"], "C", RTOL_STAT)
+    assert_rel(st["mean_sq_norm"], orc["mean_sq_norm"], "||Dbar||^2",
+               RTOL_STAT)
+    for m in range(M):
+        assert_rel(st["drift"][m], orc["drift"][m], f"||Delta_{m}||^2",
+                   RTOL_STAT)
+
+
+def assert_corr(corr: dict, oc: O.Correction):
+    for k in ("lam_sel", "lam_base", "rho_unc", "rho", "mu_t", "kappa_t",
+              "eta_out", "inv_norm"):
+        assert_rel(corr[k], getattr(oc, k), k, RTOL_SCALAR)
+
+
+def oracle_stats_threaded(g: torch.Tensor, xs, eps: float, slice_elems=1 << 24,
+                          threads: int = 16):
+    """Pass-1 sums of the oracle over a long device-resident vector: slices
+    are copied to the host and summed by oracle threads (ctypes releases the
+    GIL); the per-slice sums are then added in slice order."""
+    N = g.numel()
+    M = len(xs)
+    dt = oracle_dtype(xs[0].dtype)
+    bounds = [(s, min(N, s + slice_elems)) for s in range(0, N, slice_elems)]
+    accs = [O.Pass1Accumulator(M) for _ in bounds]
+
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        futs = []
+        for k, (s, e) in enumerate(bounds):
+            gh = g[s:e].cpu().numpy()
+            xh = [to_numpy_bits(x[s:e]) for x in xs]
+            futs.append(ex.submit(accs[k].add, gh, xh, dt))
+            if len(futs) >= 2 * threads:
+                futs.pop(0).result()
+        for f in futs:
+            f.result()
+    E = [0.0] * M
+    B = 0.0
+    for acc in accs:
+        for m in range(M):
+            E[m] += acc.E[m]
+        B += acc.B.value
+    Dsum = 0.0
+    for m in range(M):
+        Dsum += E[m]
+    D = Dsum / M
+    return {"D": D, "C": M * B / (D + eps), "mean_sq_norm": B, "drift": E}
+
+
+def sample_indices(N: int, boundaries=(), k: int = 4096, seed: int = 0):
+    """Indices to compare at full size: random ones, both ends, and the
+    first/last element of every tensor of the layout."""
+    rng = np.random.default_rng(seed)
+    idx = set(rng.integers(0, N, size=min(k, N)).tolist())
+    idx.update([0, 1, N - 2, N - 1])
+    for b in boundaries:
+        for j in (b - 1, b, b + 1):
+            if 0 <= j < N:
+                idx.add(j)
+    return torch.tensor(sorted(idx), dtype=torch.int64)
+
+
+# ------------------------------------------------------------ round runners
+
+def gpu_inputs(w: W.Workload, device="cuda", round_index=0):
+    g = W.make_global(w, device)
+    v = W.make_momentum(w, device)
+    xs = W.fill_replicas(w, g, W.alloc_replicas(w, device), round_index)
+    return g, v, xs
+
+
+def run_gpu_round(g, v, xs, w: W.Workload, step: int, H_sel: int,
+                  opts=None, stream=None):
+    sa, _ = schedule_pair(w.schedule)
+    return A.sync(g, v, xs, H_sel=H_sel, H_base=w.H_base, step=step,
+                  schedule=sa, outer_lr=w.outer_lr, outer_beta=w.outer_beta,
+                  opts=opts, stream=stream, raise_on_error=False)
+
+
+def run_oracle_round(g, v, xs, w: W.Workload, step: int, H_sel: int,
+                     normalize=False, mode=O.MODE_FULL, eps=1e-8):
+    """Oracle round on host copies (taken before the GPU overwrites them)."""
+    _, so = schedule_pair(w.schedule)
+    gh = g.cpu().numpy() if isinstance(g, torch.Tensor) else g
+    vh = v.cpu().numpy() if isinstance(v, torch.Tensor) else v
+    xh = [to_numpy_bits(x) if isinstance(x, torch.Tensor) else x for x in xs]
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+    return O.sync_round(gh, vh, xh, dt, so, step, H_sel, w.H_base, w.outer_lr,
+                        w.outer_beta, eps=eps, normalize=normalize, mode=mode)
+
+
+def compare_round(w, st, orc, g, v, xs):
+    """Element-by-element comparison of a whole round."""
+    assert st["nonfinite"] == orc["nonfinite"]
+    assert_corr(st["corr"], orc["corr"])
+    assert_stats(st, orc, w.M)
+    assert_field(g.cpu().numpy(), orc["g"], "theta'")
+    assert_field(v.cpu().numpy(), orc["v"], "v'")
+    gg = g.cpu().numpy()
+    for m, x in enumerate(xs):
+        if w.dtype == "f32":
+            xh = x.cpu().numpy()
+            assert np.array_equal(xh.view(np.uint32), gg.view(np.uint32)), \
+                f"replica {m} is not theta'"
+            assert_field(xh, orc["x"][m], f"replica {m}")
+        else:
+            bits = to_numpy_bits(x)
+            assert_bf16_is_rounded_theta(bits, g, f"replica {m}")
+            assert_bf16_replica(bits, orc["x"][m], orc["g"], f"replica {m}")
+
+
+def oracle_chain_endpoints(w: W.Workload, g_host: np.ndarray, round_index,
+                           device="cuda"):
+    """The oracle chain's own endpoints for a round: the same generator,
+    applied to the oracle's theta (uploaded chunk by chunk).  Returns the
+    fp32 values before storage and the stored replicas (fp32, or bf16 bit
+    patterns rounded to nearest even)."""
+    y = [np.empty(w.numel, np.float32) for _ in range(w.M)]
+    for c in range(W.n_chunks(w)):
+        s, e = c * W.CHUNK, min(w.numel, (c + 1) * W.CHUNK)
+        gc = torch.from_numpy(g_host[s:e]).to(device)
+        for m, x in enumerate(W.replica_chunk(w, gc, round_index, c)):
+            y[m][s:e] = x.cpu().numpy()
+    if w.dtype == "f32":
+        return y, y
+    return y, [to_bf16_bits(t) for t in y]
+
+
+def oracle_chain_replicas(w: W.Workload, g_host: np.ndarray, round_index,
+                          device="cuda"):
+    return oracle_chain_endpoints(w, g_host, round_index, device)[1]
+
+
+def to_bf16_bits(y: np.ndarray) -> np.ndarray:
+    return torch.from_numpy(np.ascontiguousarray(y, np.float32)) \
+        .to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def gather_host(t: torch.Tensor, idx: torch.Tensor) -> np.ndarray:
+    return to_numpy_bits(t[idx.to(t.device)])
+
+
+def oracle_pass2_at(w: W.Workload, g_idx, v_idx, x_idx, corr: O.Correction):
+    """The oracle's elementwise update at sampled elements (each element
+    depends only on its own inputs and the round's scalars)."""
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+    return O.pass2(g_idx, v_idx, x_idx, dt, corr.mu_t, corr.eta_out,
+                   corr.inv_norm)
+
+
+def oracle_corr(w: W.Workload, step, hsel, normalize=False, mode=O.MODE_FULL):
+    _, so = schedule_pair(w.schedule)
+    return O.correction(so, step, hsel, w.H_base, w.outer_lr, w.outer_beta,
+                        normalize=normalize, mode=mode)
+
+
+def compare_sampled(w, g_gpu_idx, v_gpu_idx, x_gpu_idx, ref,
+                    prior_rounds: int = 0):
+    """Sampled elements of a round.  In the k-th round of two independent
+    chains (prior_rounds = k) the inputs already differ by the chains' fp32
+    storage of theta; see assert_field_after_chain."""
+    g_o, v_o, x_o, _ = ref
+    if prior_rounds == 0:
+        assert_field(g_gpu_idx, g_o, "theta' (sampled)")
+        assert_field(v_gpu_idx, v_o, "v' (sampled)")
+    else:
+        assert_field_after_chain(g_gpu_idx, g_o, g_o, prior_rounds + 1,
+                                 "theta' (sampled)")
+        assert_field_after_chain(v_gpu_idx, v_o, g_o, prior_rounds + 1,
+                                 "v' (sampled)")
+    for m in range(w.M):
+        if w.dtype == "f32":
+            if prior_rounds == 0:
+                assert_field(x_gpu_idx[m], x_o[m], f"replica {m} (sampled)")
+            else:
+                assert_field_after_chain(x_gpu_idx[m], x_o[m], g_o,
+                                         prior_rounds + 1,
+                                         f"replica {m} (sampled)")
+        else:
+            assert_bf16_replica(x_gpu_idx[m], x_o[m], g_o,
+                                f"replica {m} (sampled)",
+                                extra_abs=(prior_rounds + 1) * fp32_ulp(g_o)
+                                if prior_rounds else 0.0)
+
+
+def oracle_pass2_threaded(w: W.Workload, g_h, v_h, x_h, corr,
+                          slice_elems=1 << 22, threads=16):
+    """Oracle update over whole host vectors, slices run by threads.
+    Returns fp64 theta', v'."""
+    N = g_h.shape[0]
+    g_out = np.empty(N, np.float64)
+    v_out = np.empty(N, np.float64)
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+
+    def work(s):
+        e = min(N, s + slice_elems)
+        go, vo, _, _ = O.pass2(g_h[s:e], v_h[s:e], [x[s:e] for x in x_h], dt,
+                               corr.mu_t, corr.eta_out, corr.inv_norm,
+                               want_replicas=False)
+        g_out[s:e] = go
+        v_out[s:e] = vo
+
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        list(ex.map(work, range(0, N, slice_elems)))
+    return g_out, v_out
+
+
+def oracle_stats_host_threaded(w: W.Workload, g_h, x_h, eps=1e-8,
+                               slice_elems=1 << 22, threads=16):
+    N = g_h.shape[0]
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+    starts = list(range(0, N, slice_elems))
+    accs = [O.Pass1Accumulator(w.M) for _ in starts]
+
+    def work(k):
+        s = starts[k]
+        e = min(N, s + slice_elems)
+        accs[k].add(g_h[s:e], [x[s:e] for x in x_h], dt)
+
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        list(ex.map(work, range(len(starts))))
+    E = [0.0] * w.M
+    B = 0.0
+    for acc in accs:
+        for m in range(w.M):
+            E[m] += acc.E[m]
+        B += acc.B.value
+    D = sum(E) / w.M
+    return {"D": D, "C": w.M * B / (D + eps), "mean_sq_norm": B, "drift": E}

@@ -1,0 +1,211 @@
+"""CPU-side checks of the C ABI: the library loads, exports every function
+that include/aloco.h declares, the ctypes structures match the C layout,
+and the host-only entry points (schedule mass, correction context,
+argument validation) agree with the oracle.  No GPU is needed: nothing here
+launches a kernel."""
+import ctypes
+import math
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2609_36662_gb300 import aloco as A
+from paper_2609_36662_gb300 import build as B
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "aloco.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return A.load()
+
+
+def _declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"\b(aloco_[a-z0-9_]+)\s*\(", text)
+    return sorted(set(names))
+
+
+def test_every_declared_function_is_exported(lib):
+    declared = _declared_functions()
+    assert declared, "no declarations parsed"
+    assert sorted(A.EXPORTS) == declared
+    for name in declared:
+        assert hasattr(lib, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", A.library_path()],
+                         capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (aloco_\w+)", out))
+    assert set(declared) <= exported
+
+
+def test_struct_layout_matches_c(tmp_path):
+    """Compile a probe against the public header and compare sizeof and
+    offsetof with the ctypes mirrors used by the binding."""
+    src = tmp_path / "probe.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include <stddef.h>
+#include "aloco.h"
+int main(void) {
+  printf("%zu %zu %zu %zu\n", sizeof(aloco_schedule_t), sizeof(aloco_opts_t),
+         sizeof(aloco_correction_t), sizeof(aloco_stats_t));
+  printf("%zu %zu %zu %zu %zu %zu\n", offsetof(aloco_opts_t, stream),
+         offsetof(aloco_stats_t, corr), offsetof(aloco_stats_t, nonfinite),
+         offsetof(aloco_stats_t, kernel_ms), offsetof(aloco_schedule_t, peak_lr),
+         offsetof(aloco_schedule_t, total_steps));
+  return 0;
+}
+''')
+    exe = tmp_path / "probe"
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"),
+                    str(src), "-o", str(exe)], check=True)
+    lines = subprocess.run([str(exe)], capture_output=True, text=True,
+                           check=True).stdout.split("\n")
+    sizes = list(map(int, lines[0].split()))
+    offs = list(map(int, lines[1].split()))
+    assert sizes == [ctypes.sizeof(A.Schedule), ctypes.sizeof(A.Opts),
+                     ctypes.sizeof(A.Correction), ctypes.sizeof(A.Stats)]
+    assert offs == [A.Opts.stream.offset, A.Stats.corr.offset,
+                    A.Stats.nonfinite.offset, A.Stats.kernel_ms.offset,
+                    A.Schedule.peak_lr.offset, A.Schedule.total_steps.offset]
+
+
+def test_default_opts_are_the_papers_settings(lib):
+    """Tab. AutoLoCo configuration: momentum bounds [0.45, 0.90], maximum
+    outer-step scale 1.6."""
+    o = A.default_opts()
+    assert (o.mu_min, o.mu_max, o.kappa_max) == (0.45, 0.90, 1.6)
+    assert o.eps == 1e-8 and o.normalize == 0 and o.mode == A.CORR_FULL
+    assert o.stream is None and o.time_kernel == 0
+
+
+@pytest.mark.parametrize("kind", [0, 1, 2])
+def test_lr_accum_matches_oracle(lib, kind):
+    rng = np.random.default_rng(kind)
+    sa = A.Schedule.make(kind, 4e-4, 4e-5, 1000, 40000)
+    so = O.Schedule(kind, 4e-4, 4e-5, 1000, 40000)
+    cases = [(0, 0), (0, 1), (999, 1), (999, 2), (39990, 30), (50000, 7),
+             (15000, 250), (4000, 150)]
+    cases += [(int(rng.integers(0, 45000)), int(rng.integers(0, 5000)))
+              for _ in range(100)]
+    for t0, H in cases:
+        want = O.lr_mass(so, t0, H)
+        got = A.inner_lr_accum(sa, t0, H)
+        assert got == pytest.approx(want, rel=1e-12, abs=1e-300), (t0, H)
+
+
+def test_lr_accum_rejects_bad_arguments(lib):
+    s = A.Schedule.make()
+    assert math.isnan(A.inner_lr_accum(s, -1, 5))
+    assert math.isnan(A.inner_lr_accum(s, 0, -5))
+    bad = A.Schedule.make(warmup_steps=500, total_steps=500)
+    assert math.isnan(A.inner_lr_accum(bad, 0, 5))
+    assert "warmup" in A.last_error()
+    assert math.isnan(A.inner_lr_accum(A.Schedule.make(kind=7), 0, 5))
+    assert math.isnan(A.inner_lr_accum(A.Schedule.make(peak_lr=-1.0), 0, 5))
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("normalize", [0, 1])
+def test_correction_matches_oracle(lib, mode, normalize):
+    rng = np.random.default_rng(10 * mode + normalize)
+    for _ in range(150):
+        total = int(rng.integers(2000, 60000))
+        sa = A.Schedule.make(0, 4e-4, 4e-5, 1000, total)
+        so = O.Schedule(0, 4e-4, 4e-5, 1000, total)
+        step = int(rng.integers(0, total + 1000))
+        hs, hb = int(rng.integers(1, 2000)), int(rng.integers(1, 1000))
+        eta = float(rng.uniform(0.1, 1.5))
+        beta = float(rng.uniform(0.3, 0.95))
+        opts = A.default_opts(mode=mode, normalize=normalize)
+        c = A.correction(sa, step, hs, hb, eta, beta, opts).as_dict()
+        oc = O.correction(so, step, hs, hb, eta, beta, normalize=normalize,
+                          mode=mode)
+        for k, v in c.items():
+            assert v == pytest.approx(getattr(oc, k), rel=1e-12), k
+
+
+def test_correction_argument_errors(lib):
+    s = A.Schedule.make()
+    cases = [dict(H_sel=0), dict(H_base=0), dict(step=-1),
+             dict(outer_beta=1.0), dict(outer_beta=0.0),
+             dict(outer_lr=float("nan")),
+             dict(opts=A.default_opts(eps=0.0)),
+             dict(opts=A.default_opts(mu_min=0.9, mu_max=0.5)),
+             dict(opts=A.default_opts(kappa_max=0.5)),
+             dict(opts=A.default_opts(mode=9))]
+    for kw in cases:
+        args = dict(schedule=s, step=4000, H_sel=150, H_base=100,
+                    outer_lr=0.7, outer_beta=0.9, opts=None)
+        args.update(kw)
+        with pytest.raises(A.AlocoError) as ei:
+            A.correction(**args)
+        assert ei.value.status == A.ERR_ARG, kw
+    # beta = 0 is allowed without correction (direct averaging)
+    A.correction(s, 4000, 150, 100, 1.0, 0.0, A.default_opts(mode=A.CORR_NONE))
+
+
+def test_sync_argument_errors_before_any_device_work(lib):
+    """Validation happens before the library touches CUDA: fake addresses
+    are never dereferenced."""
+    s = A.Schedule.make()
+    base = 1 << 40
+    xs = [base + (k + 2) * (1 << 20) for k in range(4)]
+    rc, _ = A.sync_ptrs(base, base + (1 << 20), xs, 1000, A.F32, 150, 100,
+                        4000, s, 0.7, 0.9, raise_on_error=False)
+    assert rc in (A.ERR_CUDA, A.ERR_ARG)   # no device here
+    # M out of range
+    rc, _ = A.sync_ptrs(base, base + 8192, [], 10, A.F32, 150, 100, 4000, s,
+                        0.7, 0.9, raise_on_error=False)
+    assert rc == A.ERR_ARG
+    rc, _ = A.sync_ptrs(base, base + 8192, [base + 16384 * (k + 1)
+                                            for k in range(33)],
+                        10, A.F32, 150, 100, 4000, s, 0.7, 0.9,
+                        raise_on_error=False)
+    assert rc == A.ERR_ARG
+    # overlapping replica and global
+    rc, _ = A.sync_ptrs(base, base + (1 << 20), [base + 64], 1000, A.F32,
+                        150, 100, 4000, s, 0.7, 0.9, raise_on_error=False)
+    assert rc == A.ERR_ALIAS and "overlap" in A.last_error()
+    # two replicas that overlap
+    rc, _ = A.sync_ptrs(base, base + (1 << 20), [base + (2 << 20),
+                                                 base + (2 << 20) + 400],
+                        1000, A.BF16, 150, 100, 4000, s, 0.7, 0.9,
+                        raise_on_error=False)
+    assert rc == A.ERR_ALIAS
+    # misaligned fp32 buffer
+    rc, _ = A.sync_ptrs(base + 2, base + (1 << 20), [base + (2 << 20)], 1000,
+                        A.F32, 150, 100, 4000, s, 0.7, 0.9,
+                        raise_on_error=False)
+    assert rc == A.ERR_ARG
+    # bad horizons / dtype / NULL
+    for kw in (dict(H_sel=0), dict(H_base=-3), dict(dtype=5)):
+        a = dict(g_ptr=base, v_ptr=base + (1 << 20), x_ptrs=[base + (2 << 20)],
+                 N=100, dtype=A.F32, H_sel=150, H_base=100, step=4000,
+                 schedule=s, outer_lr=0.7, outer_beta=0.9,
+                 raise_on_error=False)
+        a.update(kw)
+        rc, _ = A.sync_ptrs(**a)
+        assert rc == A.ERR_ARG, kw
+    rc, _ = A.sync_ptrs(0, base, [base + (2 << 20)], 100, A.F32, 150, 100,
+                        4000, s, 0.7, 0.9, raise_on_error=False)
+    assert rc == A.ERR_ARG
+
+
+def test_empty_round_needs_no_device(lib):
+    """N = 0 is a valid round: no kernel runs, the statistics are zero and
+    the correction context is still reported."""
+    s = A.Schedule.make()
+    rc, st = A.sync_ptrs(0, 0, [0, 0], 0, A.F32, 150, 100, 4000, s, 0.7, 0.9)
+    assert rc == A.OK
+    d = st.as_dict()
+    assert d["D"] == 0.0 and d["C"] == 0.0 and d["nonfinite"] == 0
+    oc = O.correction(O.Schedule(), 4000, 150, 100, 0.7, 0.9)
+    assert d["corr"]["rho"] == pytest.approx(oc.rho, rel=1e-12)

@@ -1,0 +1,281 @@
+"""Parity of the CUDA round (through the C ABI) with the fp64 oracle on the
+same seeded inputs, at sizes the oracle finishes in seconds: several
+thousand blocks' worth of packs, ragged tails, unaligned buffers, every
+worker count from 1 to 32, both replica types, all correction modes."""
+import glob
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2609_36662_gb300 import aloco as A
+from paper_2609_36662_gb300 import workloads as W
+
+from _parity import (assert_corr, assert_field, assert_field_after_chain,
+                     assert_stats, compare_round, gpu_inputs,
+                     oracle_chain_replicas,
+                     run_gpu_round, run_oracle_round, schedule_pair,
+                     to_numpy_bits)
+
+pytestmark = pytest.mark.gpu
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    yield
+    A.shutdown()
+
+
+@pytest.mark.parametrize("path", sorted(glob.glob(os.path.join(
+    GOLDEN, "dyadic_round_*.json"))))
+@pytest.mark.parametrize("rdt", [torch.float32, torch.bfloat16])
+def test_hand_worked_rounds_bit_exact(path, rdt):
+    """Dyadic inputs make every fp32 step exact: the GPU must reproduce the
+    hand-worked values bit for bit."""
+    fx = json.load(open(path))
+    g = torch.tensor(fx["g"], dtype=torch.float32, device="cuda")
+    v = torch.tensor(fx["v"], dtype=torch.float32, device="cuda")
+    xs = [torch.tensor(x, dtype=torch.float32, device="cuda").to(rdt)
+          for x in fx["x"]]
+    mode = {"none": A.CORR_NONE, "full": A.CORR_FULL}[fx["mode"]]
+    st = A.sync(g, v, xs, H_sel=fx["H_sel"], H_base=fx["H_base"], step=4000,
+                schedule=A.Schedule.make(), outer_lr=fx["eta"],
+                outer_beta=fx["mu"], opts=A.default_opts(mode=mode))
+    ex = fx["expect"]
+    assert st["status"] == A.OK
+    assert g.cpu().tolist() == ex["g"]
+    assert v.cpu().tolist() == ex["v"]
+    for x in xs:
+        assert x.float().cpu().tolist() == ex["g"]
+    assert st["drift"] == ex["drift"]
+    assert st["mean_sq_norm"] == ex["mean_sq_norm"]
+    assert st["D"] == ex["D"]
+    assert st["C"] == pytest.approx(ex["C_numerator"] / (ex["D"] + 1e-8),
+                                    rel=1e-15)
+
+
+SMALL = [(n, m, dt) for n in (1, 7, 4097) for m in (1, 2, 3, 5, 8, 13, 16,
+                                                    17, 32)
+         for dt in ("f32", "bf16")]
+MEDIUM = [(1_000_003, m, dt) for m in (1, 3, 4, 8, 16, 17, 32)
+          for dt in ("f32", "bf16")]
+
+
+@pytest.mark.parametrize("N,M,dt", SMALL + MEDIUM)
+def test_round_matches_oracle(N, M, dt):
+    w = W.small(N, M, dt, seed=N % 97 + M)
+    g, v, xs = gpu_inputs(w)
+    v.normal_(0, 1e-3)          # carried momentum
+    orc = run_oracle_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    assert st["status"] == A.OK
+    compare_round(w, st, orc, g, v, xs)
+
+
+def test_toy_round_matches_oracle():
+    """The 2^20-parameter, 4-worker fp32 round at step 4000 (H_sel 150,
+    H_base 100, cosine 4e-4 -> 4e-5 over 20000 steps)."""
+    w = W.toy_round()
+    g, v, xs = gpu_inputs(w)
+    orc = run_oracle_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    assert st["status"] == A.OK
+    compare_round(w, st, orc, g, v, xs)
+    assert st["corr"]["rho"] == pytest.approx(1.4985573577339066, rel=1e-12)
+
+
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+@pytest.mark.parametrize("offset", [1, 2, 3])
+def test_unaligned_buffers(dt, offset):
+    """Buffers that are not 16-byte aligned take the element-wise path."""
+    N, M = 100_003, 5
+    w = W.small(N + 8, M, dt, seed=offset)
+    g0, v0, xs0 = gpu_inputs(w)
+    g, v = g0[offset:offset + N], v0[offset + 1:offset + 1 + N]
+    xs = [x[offset:offset + N] for x in xs0]
+    wN = W.small(N, M, dt, seed=offset)
+    orc = run_oracle_round(g, v, xs, wN, wN.start_step, wN.H_sel[0])
+    st = run_gpu_round(g, v, xs, wN, wN.start_step, wN.H_sel[0])
+    assert st["status"] == A.OK
+    compare_round(wN, st, orc, g, v, xs)
+
+
+@pytest.mark.parametrize("mode", [A.CORR_FULL, A.CORR_MOMENTUM_ONLY,
+                                  A.CORR_NONE])
+@pytest.mark.parametrize("normalize", [0, 1])
+def test_modes_and_normalisation(mode, normalize):
+    w = W.small(300_001, 6, "f32", seed=3, H_sel=400, H_base=100)
+    g, v, xs = gpu_inputs(w)
+    v.normal_(0, 1e-3)
+    orc = run_oracle_round(g, v, xs, w, 9000, 400, normalize=bool(normalize),
+                           mode=mode)
+    st = run_gpu_round(g, v, xs, w, 9000, 400,
+                       opts=A.default_opts(mode=mode, normalize=normalize))
+    compare_round(w, st, orc, g, v, xs)
+
+
+def test_direct_averaging_gives_the_mean_of_endpoints():
+    """No momentum, unit outer lr, no correction: theta' is the average of
+    the workers' endpoints (the baselines' direct model averaging)."""
+    w = W.small(65_537, 4, "f32", seed=12)
+    g, v, xs = gpu_inputs(w)
+    mean = torch.stack([x.double() for x in xs]).mean(0)
+    sa, _ = schedule_pair(w.schedule)
+    A.sync(g, v, xs, H_sel=100, H_base=100, step=0, schedule=sa, outer_lr=1.0,
+           outer_beta=0.0, opts=A.default_opts(mode=A.CORR_NONE))
+    assert_field(g.cpu().numpy(), mean.cpu().numpy(), "mean")
+
+
+def test_repeated_rounds_are_bit_identical():
+    w = W.small(2_000_003, 8, "bf16", seed=5)
+    results = []
+    for _ in range(5):
+        g, v, xs = gpu_inputs(w)
+        v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(1))
+        st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0])
+        results.append((st["D"], st["C"], tuple(st["drift"]),
+                        st["mean_sq_norm"], g.cpu().numpy().tobytes(),
+                        v.cpu().numpy().tobytes(),
+                        to_numpy_bits(xs[3]).tobytes()))
+    assert all(r == results[0] for r in results[1:])
+
+
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+def test_guard_bands_untouched(dt):
+    """Only [0, N) of each buffer is written: 64 sentinel elements on both
+    sides of every buffer stay intact."""
+    N, M, pad = 123_457, 3, 64
+    w = W.small(N, M, dt, seed=9)
+    g, v, xs = gpu_inputs(w)
+    def padded(t, fill):
+        big = torch.full((N + 2 * pad,), fill, dtype=t.dtype, device="cuda")
+        big[pad:pad + N] = t
+        return big
+    gb, vb = padded(g, 7.0), padded(v, -7.0)
+    xb = [padded(x, 3.0) for x in xs]
+    st = run_gpu_round(gb[pad:pad + N], vb[pad:pad + N],
+                       [x[pad:pad + N] for x in xb], w, w.start_step,
+                       w.H_sel[0])
+    assert st["status"] == A.OK
+    for t, fill in [(gb, 7.0), (vb, -7.0)] + [(x, 3.0) for x in xb]:
+        assert torch.all(t[:pad] == fill) and torch.all(t[-pad:] == fill)
+
+
+def test_nonfinite_inputs_are_reported():
+    """NaN/Inf in the inputs propagate through the round; the status says so
+    and the count of affected elements matches the oracle's."""
+    w = W.small(50_000, 4, "f32", seed=21)
+    g, v, xs = gpu_inputs(w)
+    xs[1][100] = float("nan")
+    xs[2][100] = float("inf")
+    v[4000] = float("inf")
+    g[49_999] = float("nan")
+    xs[0][777] = float("-inf")
+    orc = run_oracle_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    assert st["status"] == A.ERR_NONFINITE
+    assert st["nonfinite"] == orc["nonfinite"] == 4
+    assert "non-finite" in A.last_error()
+    # the remaining elements are still updated like the oracle's
+    mask = np.ones(50_000, bool)
+    mask[[100, 4000, 49_999, 777]] = False
+    assert_field(g.cpu().numpy()[mask], orc["g"][mask], "theta'")
+
+
+def test_host_memory_is_rejected():
+    w = W.small(1000, 2, "f32")
+    g, v, xs = gpu_inputs(w)
+    host = torch.zeros(1000, dtype=torch.float32)
+    sa, _ = schedule_pair(w.schedule)
+    rc, _ = A.sync_ptrs(host.data_ptr(), v.data_ptr(),
+                        [x.data_ptr() for x in xs], 1000, A.F32, 150, 100,
+                        4000, sa, 0.7, 0.9, raise_on_error=False)
+    assert rc == A.ERR_ARG and "device memory" in A.last_error()
+    assert torch.all(host == 0)
+
+
+def test_side_stream_and_kernel_timing():
+    w = W.small(4_000_000, 4, "bf16", seed=2)
+    g, v, xs = gpu_inputs(w)
+    orc = run_oracle_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    s = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0],
+                       opts=A.default_opts(time_kernel=1), stream=s)
+    assert st["kernel_ms"] > 0.0
+    compare_round(w, st, orc, g, v, xs)
+
+
+def _chain_workload(dt):
+    base = W.llama_150m()
+    return W.Workload("chain", 600_011, 8, dt, None, 0.6, 0.8, 1e-3, False,
+                      base.schedule, base.start_step, base.H_base, base.H_sel,
+                      7)
+
+
+def test_consecutive_rounds_track_an_independent_oracle_chain():
+    """Twenty fp32 rounds with momentum carried across them and horizons
+    drawn by seed; each round's endpoints are drawn around the chain's own
+    theta (workers restart from the synchronised model, Algorithm 1).  The
+    oracle runs its own chain -- theta and v stored in fp32 between rounds,
+    like the paper's FP32 master weights and outer state -- and nothing of
+    the GPU chain enters it.  The final state allows for the two chains'
+    independent fp32 storage of theta."""
+    w = _chain_workload("f32")
+    g, v, xs = gpu_inputs(w)
+    g_o = g.cpu().numpy().copy()
+    v_o = v.cpu().numpy().copy()
+    rounds = W.steps_of_rounds(w)
+    for k, (step, hsel) in enumerate(rounds):
+        if k > 0:
+            W.fill_replicas(w, g, xs, k)
+        x_o = oracle_chain_replicas(w, g_o, k)
+        orc = run_oracle_round(g_o, v_o, x_o, w, step, hsel)
+        st = run_gpu_round(g, v, xs, w, step, hsel)
+        assert st["status"] == A.OK
+        assert_corr(st["corr"], orc["corr"])
+        assert_stats(st, orc, w.M)
+        g_o = orc["g"].astype(np.float32)
+        v_o = orc["v"].astype(np.float32)
+    R = len(rounds)
+    assert_field_after_chain(g.cpu().numpy(), orc["g"], orc["g"], R,
+                             "theta after 20 rounds")
+    assert_field_after_chain(v.cpu().numpy(), orc["v"], orc["g"], R,
+                             "v after 20 rounds")
+
+
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+def test_momentum_carried_across_rounds(dt):
+    """Twenty rounds that carry the outer momentum while theta and the
+    endpoints are drawn afresh from the seed every round, so both sides see
+    bit-identical theta and endpoints and only v is each side's own state.
+    The momentum recurrence contracts (mu_t < 1), so the two chains' v stay
+    within the per-round tolerance; D_t and C_t are compared at 1e-6 in
+    every round.  (With bf16 endpoints around a carried fp32 theta the
+    pseudo-gradient would contain theta's sub-bf16 bits, and the outer step
+    would amplify any rounding difference between two chains by
+    |1 - eta_out (1 + mu_t)| per round.)"""
+    w = _chain_workload(dt)
+    v = W.make_momentum(w, "cuda")
+    xs = W.alloc_replicas(w, "cuda")
+    v_o = v.cpu().numpy().copy()
+    for k, (step, hsel) in enumerate(W.steps_of_rounds(w)):
+        g = W.make_global(w, "cuda", draw=k)
+        W.fill_replicas(w, g, xs, k)
+        orc = run_oracle_round(g, v_o, xs, w, step, hsel)
+        st = run_gpu_round(g, v, xs, w, step, hsel)
+        assert st["status"] == A.OK
+        assert_corr(st["corr"], orc["corr"])
+        assert_stats(st, orc, w.M)
+        assert_field(g.cpu().numpy(), orc["g"], f"theta' round {k}")
+        assert_field(v.cpu().numpy(), orc["v"], f"v' round {k}")
+        v_o = orc["v"].astype(np.float32)
