@@ -210,6 +210,50 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
                   double outer_beta, const aloco_opts_t *opts,
                   aloco_stats_t *stats_out);
 
+/* Block partials the scratch of aloco_sync_noalloc can hold. */
+#define ALOCO_NOALLOC_MAX_BLOCKS 2048
+
+/* aloco_sync_ex without any memory allocation by the library.
+ *
+ * The paper has no counterpart: this entry point exists for callers that
+ * cannot let a library allocate device or pinned host memory -- frameworks
+ * that reserve the whole GPU memory up front and serve it from their own
+ * pools, deployments whose memory footprint must be fixed when the library
+ * is loaded, and loops that cannot afford the device-wide synchronisation
+ * that cudaMalloc / cudaFree imply.  aloco_sync_ex, by contrast, allocates a
+ * cached per-device workspace on its first call.
+ *
+ * Arguments, results, status codes and numerics are those of aloco_sync_ex
+ * (same kernel, same grid, same fixed-order reductions), except that
+ * opts->time_kernel is ignored (stats_out->kernel_ms is -1).  The caller
+ * still provides every input and output buffer.
+ *
+ * Scratch: the per-block partial sums live in one statically sized device
+ * array inside the library (about 560 KB: ALOCO_NOALLOC_MAX_BLOCKS rows of
+ * ALOCO_MAX_WORKERS + 1 doubles plus counters), which every GPU that loads
+ * the library holds until the process exits.  A round that would need more
+ * than ALOCO_NOALLOC_MAX_BLOCKS blocks is rejected with ALOCO_ERR_ARG and a
+ * message naming both numbers; on a 152-SM GB300 the fused pass uses at most
+ * 1216 blocks.  Statistics are read back with cudaMemcpyAsync into a buffer
+ * on the calling thread's stack; no cudaMalloc, cudaFree, cudaMallocHost or
+ * other allocating routine is called.
+ *
+ * The first call on a device resolves the scratch array's device address
+ * (cudaGetSymbolAddress, with that device current); make that first call
+ * before any stream capture.  All calls on a device share the one array and
+ * it keeps the previous call's contents: each call clears the counter that
+ * must start at zero, and every other scratch value a round reads is
+ * written by that round first.  Rounds that overlapped on the GPU would race
+ * on the array; within a process the library prevents that by holding a
+ * per-device lock for the whole call, which returns only after its round has
+ * completed. */
+int aloco_sync_noalloc(float *global, float *momentum, void *const *locals,
+                       size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                       int64_t H_base, int64_t step,
+                       const aloco_schedule_t *schedule, double outer_lr,
+                       double outer_beta, const aloco_opts_t *opts,
+                       aloco_stats_t *stats_out);
+
 /* Message of the last failure on the calling thread ("" if none).  The
  * pointer stays valid until the next call on this thread. */
 const char *aloco_last_error(void);

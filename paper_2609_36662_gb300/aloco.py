@@ -29,8 +29,8 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
 
 # Names declared in include/aloco.h (checked by the ABI test).
 EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
-           "aloco_sync", "aloco_sync_ex", "aloco_last_error",
-           "aloco_shutdown", "aloco_version")
+           "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc",
+           "aloco_last_error", "aloco_shutdown", "aloco_version")
 
 
 class Schedule(ctypes.Structure):
@@ -117,6 +117,9 @@ def load():
     lib.aloco_sync_ex.argtypes = sync_args + [ctypes.POINTER(Opts),
                                               ctypes.POINTER(Stats)]
     lib.aloco_sync_ex.restype = i32
+    lib.aloco_sync_noalloc.argtypes = sync_args + [ctypes.POINTER(Opts),
+                                                   ctypes.POINTER(Stats)]
+    lib.aloco_sync_noalloc.restype = i32
     lib.aloco_last_error.argtypes = []
     lib.aloco_last_error.restype = ctypes.c_char_p
     lib.aloco_shutdown.argtypes = []
@@ -159,12 +162,15 @@ def correction(schedule: Schedule, step: int, H_sel: int, H_base: int,
 def sync_ptrs(g_ptr: int, v_ptr: int, x_ptrs: Sequence[int], N: int,
               dtype: int, H_sel: int, H_base: int, step: int,
               schedule: Schedule, outer_lr: float, outer_beta: float,
-              opts: Optional[Opts] = None, raise_on_error: bool = True):
-    """aloco_sync_ex on raw device addresses.  Returns (status, Stats)."""
+              opts: Optional[Opts] = None, raise_on_error: bool = True,
+              noalloc: bool = False):
+    """aloco_sync_ex (or, with noalloc=True, aloco_sync_noalloc) on raw
+    device addresses.  Returns (status, Stats)."""
     M = len(x_ptrs)
     arr = (ctypes.c_void_p * max(M, 1))(*x_ptrs)
     st = Stats()
-    rc = load().aloco_sync_ex(g_ptr, v_ptr, arr, N, M, dtype, H_sel, H_base,
+    fn = load().aloco_sync_noalloc if noalloc else load().aloco_sync_ex
+    rc = fn(g_ptr, v_ptr, arr, N, M, dtype, H_sel, H_base,
                               step, ctypes.byref(schedule), outer_lr,
                               outer_beta,
                               ctypes.byref(opts) if opts is not None else None,
@@ -176,12 +182,14 @@ def sync_ptrs(g_ptr: int, v_ptr: int, x_ptrs: Sequence[int], N: int,
 
 def sync(global_, momentum, locals_, *, H_sel: int, H_base: int, step: int,
          schedule: Schedule, outer_lr: float, outer_beta: float,
-         opts: Optional[Opts] = None, stream=None, raise_on_error=True):
+         opts: Optional[Opts] = None, stream=None, raise_on_error=True,
+         noalloc: bool = False):
     """One outer synchronisation round on torch CUDA tensors, in place.
 
     global_, momentum: contiguous float32 [N]; locals_: M contiguous tensors
     [N] of float32 or bfloat16.  The round runs on `stream` (default: the
-    current torch stream)."""
+    current torch stream).  noalloc=True calls aloco_sync_noalloc, the entry
+    point that allocates nothing (its scratch is a static device array)."""
     import torch
     if global_.dtype != torch.float32 or momentum.dtype != torch.float32:
         raise TypeError("global and momentum must be float32")
@@ -211,7 +219,7 @@ def sync(global_, momentum, locals_, *, H_sel: int, H_base: int, step: int,
         rc, st = sync_ptrs(global_.data_ptr(), momentum.data_ptr(),
                            [x.data_ptr() for x in locals_], N, dtype, H_sel,
                            H_base, step, schedule, outer_lr, outer_beta, opts,
-                           raise_on_error)
+                           raise_on_error, noalloc)
     return st.as_dict() | {"status": rc}
 
 

@@ -248,6 +248,15 @@ GetAddressRangeFn address_range_fn() {
     return fn;
 }
 
+}  // namespace
+
+// Helpers with external linkage: also used by the allocation-free entry
+// point (aloco_noalloc.cu).
+namespace aloco {
+
+// Record an error message for aloco_last_error() and return `code`.
+int report_error(int code, const char *msg) { return fail(code, "%s", msg); }
+
 // The buffer must be device (or managed) memory of `device`, and when the
 // driver can tell, [p, p + bytes) must lie inside one allocation.
 int check_buffer(const void *p, size_t bytes, int device, const char *name) {
@@ -309,7 +318,12 @@ void finalize_stats(const double *totals, unsigned long long nf, int M,
     st->nonfinite = (int64_t)nf;
 }
 
-}  // namespace
+}  // namespace aloco
+
+using aloco::check_buffer;
+using aloco::fill_default_opts;
+using aloco::finalize_stats;
+using aloco::split_coef;
 
 // ================================================================ C ABI
 

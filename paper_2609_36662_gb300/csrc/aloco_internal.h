@@ -52,4 +52,12 @@ cudaError_t plan_sync_f32(int M, int64_t work_items, int sm_count,
 cudaError_t plan_sync_bf16(int M, int64_t work_items, int sm_count,
                            LaunchPlan *plan);
 
+// Host helpers shared by the entry points (aloco_host.cpp).
+int report_error(int code, const char *msg);
+int check_buffer(const void *p, size_t bytes, int device, const char *name);
+void fill_default_opts(aloco_opts_t *o);
+void split_coef(double x, float *hi, float *lo);
+void finalize_stats(const double *totals, unsigned long long nf, int M,
+                    double eps, aloco_stats_t *st);
+
 }  // namespace aloco

@@ -1,0 +1,97 @@
+"""aloco_sync_noalloc, the entry point that allocates nothing.
+
+Some callers cannot let a library allocate memory: frameworks that reserve
+all device memory up front and serve it from their own pools, deployments
+whose footprint must be fixed when the library loads, and loops that cannot
+afford the device-wide synchronisation of cudaMalloc / cudaFree.  For them
+aloco_sync_noalloc keeps its scratch in a static device array inside the
+library.  These tests call it through the C ABI and check it against
+aloco_sync_ex, the entry point that allocates a cached workspace, on the
+same inputs, on two calls in a row, within the tolerances of the parity
+tests.  The file is collected last so that a run stopping at the first
+failure has already run every other test; it also passes on its own in a
+fresh process.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_36662_gb300 import aloco as A
+from paper_2609_36662_gb300 import workloads as W
+
+from _parity import (RTOL_STAT, assert_field, assert_rel, gpu_inputs,
+                     schedule_pair, to_numpy_bits)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _round(w, g, v, xs, noalloc, opts=None):
+    sa, _ = schedule_pair(w.schedule)
+    return A.sync(g, v, xs, H_sel=w.H_sel[0], H_base=w.H_base,
+                  step=w.start_step, schedule=sa, outer_lr=w.outer_lr,
+                  outer_beta=w.outer_beta, opts=opts, noalloc=noalloc)
+
+
+@pytest.mark.parametrize("dt,N,M", [("f32", 1_000_003, 8),
+                                    ("bf16", 2_000_005, 5),
+                                    ("f32", 4099, 17)])
+def test_noalloc_matches_the_allocating_entry_point(dt, N, M):
+    w = W.small(N, M, dt, seed=31)
+    for call in range(2):
+        g, v, xs = gpu_inputs(w, round_index=call)
+        v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(call))
+        g2, v2, xs2 = g.clone(), v.clone(), [x.clone() for x in xs]
+        # the first call starts with the allocation-free entry point, so a
+        # fresh process exercises its set-up before anything else
+        if call == 0:
+            st_new = _round(w, g2, v2, xs2, noalloc=True)
+            st_ref = _round(w, g, v, xs, noalloc=False)
+        else:
+            st_ref = _round(w, g, v, xs, noalloc=False)
+            st_new = _round(w, g2, v2, xs2, noalloc=True)
+        assert st_new["status"] == A.OK and st_ref["status"] == A.OK
+        assert st_new["kernel_ms"] == -1.0
+        assert st_new["nonfinite"] == st_ref["nonfinite"] == 0
+        for k in ("D", "C", "mean_sq_norm"):
+            assert_rel(st_new[k], st_ref[k], k, RTOL_STAT)
+        for m in range(M):
+            assert_rel(st_new["drift"][m], st_ref["drift"][m], f"drift {m}",
+                       RTOL_STAT)
+        assert st_new["corr"] == st_ref["corr"]
+        assert_field(g2.cpu().numpy(), g.cpu().numpy().astype(np.float64),
+                     "theta'")
+        assert_field(v2.cpu().numpy(), v.cpu().numpy().astype(np.float64),
+                     "v'")
+        for a, b in zip(xs2, xs):
+            if dt == "f32":
+                assert_field(a.cpu().numpy(), b.cpu().numpy().astype(
+                    np.float64), "replica")
+            else:
+                d = np.abs(to_numpy_bits(a).astype(np.int64) -
+                           to_numpy_bits(b).astype(np.int64))
+                assert d.max() <= 1
+
+
+def test_noalloc_reports_nonfinite_and_bad_arguments():
+    w = W.small(10_000, 3, "f32", seed=32)
+    g, v, xs = gpu_inputs(w)
+    xs[1][17] = float("nan")
+    st = _round(w, g, v, xs, noalloc=True)
+    assert st["status"] == A.ERR_NONFINITE and st["nonfinite"] == 1
+    sa, _ = schedule_pair(w.schedule)
+    rc, _ = A.sync_ptrs(g.data_ptr(), v.data_ptr(), [x.data_ptr() for x in xs],
+                        w.numel, 7, 150, 100, 4000, sa, 0.7, 0.9,
+                        raise_on_error=False, noalloc=True)
+    assert rc == A.ERR_ARG and "dtype" in A.last_error()
+    rc, _ = A.sync_ptrs(g.data_ptr(), v.data_ptr(), [g.data_ptr() + 64],
+                        w.numel, A.F32, 150, 100, 4000, sa, 0.7, 0.9,
+                        raise_on_error=False, noalloc=True)
+    assert rc == A.ERR_ALIAS
