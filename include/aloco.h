@@ -107,8 +107,8 @@ typedef enum {
 
 /* Options.  aloco_default_opts() fills the paper's settings
  * (Tab. AutoLoCo configuration): mu_min 0.45, mu_max 0.90, kappa_max 1.6,
- * eps 1e-8, normalize off, FULL correction, no kernel timing, default
- * stream.  Passing NULL where an opts pointer is accepted means these
+ * eps 1e-8, normalize off, FULL correction, no kernel timing, the tuned
+ * launch configuration, default stream.  Passing NULL where an opts pointer is accepted means these
  * defaults. */
 typedef struct aloco_opts {
     double mu_min;
@@ -119,7 +119,12 @@ typedef struct aloco_opts {
     int32_t mode;         /* aloco_corr_mode                                 */
     int32_t time_kernel;  /* 1: stats_out->kernel_ms = duration of the fused
                              pass, from CUDA events on the launch stream     */
-    int32_t reserved;
+    int32_t blocks_per_sm;/* resident blocks per SM of the fused pass; 0 =
+                             the library's tuned choice for (M, dtype).  It
+                             is capped at what the kernel's registers allow.
+                             The grid fixes the order of the fp64 partial
+                             sums, so a different value can change the
+                             statistics in their last bits.                  */
     void *stream;         /* cudaStream_t; NULL = legacy default stream      */
 } aloco_opts_t;
 

@@ -49,7 +49,8 @@ class Opts(ctypes.Structure):
     _fields_ = [("mu_min", ctypes.c_double), ("mu_max", ctypes.c_double),
                 ("kappa_max", ctypes.c_double), ("eps", ctypes.c_double),
                 ("normalize", ctypes.c_int32), ("mode", ctypes.c_int32),
-                ("time_kernel", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("time_kernel", ctypes.c_int32),
+                ("blocks_per_sm", ctypes.c_int32),
                 ("stream", ctypes.c_void_p)]
 
 

@@ -52,23 +52,31 @@ def up_to_date() -> bool:
     return all(os.path.getmtime(d) <= t for d in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
-    if not force and up_to_date():
+def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False,
+          out: str = None, defines=()) -> str:
+    """Compile and link the library.  `out` and `defines` (e.g.
+    ("ALOCO_UNROLL=2",)) build a variant with other tuning knobs into
+    another file; the default build uses the knobs' defaults."""
+    lib_path = out or LIB
+    if not force and out is None and not defines and up_to_date():
         return LIB
     cuda = _cuda_home()
     nvcc = os.path.join(cuda, "bin", "nvcc")
-    os.makedirs(OBJ_DIR, exist_ok=True)
+    obj_dir = OBJ_DIR if out is None else lib_path + ".objs"
+    os.makedirs(obj_dir, exist_ok=True)
     cu, cpp = _sources()
     jobs = []
+    dflags = [f"-D{d}" for d in defines]
     for src in cu:
-        obj = os.path.join(OBJ_DIR, os.path.basename(src) + ".o")
-        cmd = [nvcc, *ARCH, *NVCC_FLAGS, "-I", INCLUDE, "-c", src, "-o", obj]
+        obj = os.path.join(obj_dir, os.path.basename(src) + ".o")
+        cmd = [nvcc, *ARCH, *NVCC_FLAGS, *dflags, "-I", INCLUDE, "-c", src,
+               "-o", obj]
         if ptxas_info:
             cmd[1:1] = ["-Xptxas", "-v"]
         jobs.append((cmd, obj))
     for src in cpp:
-        obj = os.path.join(OBJ_DIR, os.path.basename(src) + ".o")
-        cmd = ["g++", *CXX_FLAGS, "-I", INCLUDE, "-I",
+        obj = os.path.join(obj_dir, os.path.basename(src) + ".o")
+        cmd = ["g++", *CXX_FLAGS, *dflags, "-I", INCLUDE, "-I",
                os.path.join(cuda, "include"), "-c", src, "-o", obj]
         jobs.append((cmd, obj))
 
@@ -88,15 +96,15 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
         for log in logs:
             if log:
                 print(log, file=sys.stderr)
-    tmp = LIB + ".tmp%d" % os.getpid()
+    tmp = lib_path + ".tmp%d" % os.getpid()
     link = [nvcc, *ARCH, "-shared", "-o", tmp,
             *[obj for _, obj in jobs], "-cudart", "static"]
     r = subprocess.run(link, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n" + " ".join(link) + "\n" +
                            r.stdout + r.stderr)
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":

@@ -108,6 +108,8 @@ int correction_impl(const aloco_schedule_t *sched, int64_t step,
                     (long long)H_sel, (long long)H_base);
     if (step < 0) return fail(ALOCO_ERR_ARG, "step must be >= 0");
     if (!std::isfinite(outer_lr)) return fail(ALOCO_ERR_ARG, "outer_lr must be finite");
+    if (o.blocks_per_sm < 0)
+        return fail(ALOCO_ERR_ARG, "blocks_per_sm must be >= 0");
     if (o.mode != ALOCO_CORR_FULL && o.mode != ALOCO_CORR_MOMENTUM_ONLY &&
         o.mode != ALOCO_CORR_NONE)
         return fail(ALOCO_ERR_ARG, "unknown correction mode %d", o.mode);
@@ -295,6 +297,7 @@ void fill_default_opts(aloco_opts_t *o) {
     o->normalize = 0;
     o->mode = ALOCO_CORR_FULL;
     o->time_kernel = 0;
+    o->blocks_per_sm = 0;
     o->stream = nullptr;
 }
 
@@ -460,8 +463,8 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
 
     const int64_t work = a.nvec > 0 ? a.nvec : a.n;
     aloco::LaunchPlan plan;
-    e = dtype == ALOCO_F32 ? aloco::plan_sync_f32(M, work, ws->sm_count, &plan)
-                           : aloco::plan_sync_bf16(M, work, ws->sm_count, &plan);
+    e = dtype == ALOCO_F32 ? aloco::plan_sync_f32(M, work, ws->sm_count, o.blocks_per_sm, &plan)
+                           : aloco::plan_sync_bf16(M, work, ws->sm_count, o.blocks_per_sm, &plan);
     if (e != cudaSuccess) return cuda_fail(e, "launch plan");
     if (plan.grid > ws->max_grid)
         return fail(ALOCO_ERR_CUDA, "grid %d exceeds workspace %d", plan.grid,

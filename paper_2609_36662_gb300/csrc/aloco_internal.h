@@ -47,10 +47,12 @@ struct LaunchPlan {
 };
 
 // Pick the kernel instance and grid; returns cudaSuccess or an error.
+// blocks_per_sm = 0 takes the tuned residency for (M, dtype); any other
+// value is used as given, capped by the kernel's occupancy limit.
 cudaError_t plan_sync_f32(int M, int64_t work_items, int sm_count,
-                          LaunchPlan *plan);
+                          int blocks_per_sm, LaunchPlan *plan);
 cudaError_t plan_sync_bf16(int M, int64_t work_items, int sm_count,
-                           LaunchPlan *plan);
+                           int blocks_per_sm, LaunchPlan *plan);
 
 // Host helpers shared by the entry points (aloco_host.cpp).
 int report_error(int code, const char *msg);

@@ -177,8 +177,8 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
     const int64_t work = a.nvec > 0 ? a.nvec : a.n;
     aloco::LaunchPlan plan;
     e = dtype == ALOCO_F32
-            ? aloco::plan_sync_f32(M, work, g_sms[device], &plan)
-            : aloco::plan_sync_bf16(M, work, g_sms[device], &plan);
+            ? aloco::plan_sync_f32(M, work, g_sms[device], o.blocks_per_sm, &plan)
+            : aloco::plan_sync_bf16(M, work, g_sms[device], o.blocks_per_sm, &plan);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return errf(ALOCO_ERR_CUDA, "launch plan: %s", cudaGetErrorString(e));

@@ -3,7 +3,7 @@
 
 namespace aloco {
 cudaError_t plan_sync_f32(int M, int64_t work_items, int sm_count,
-                          LaunchPlan *plan) {
-    return plan_dispatch<false>(M, work_items, sm_count, plan);
+                          int blocks_per_sm, LaunchPlan *plan) {
+    return plan_dispatch<false>(M, work_items, sm_count, blocks_per_sm, plan);
 }
 }  // namespace aloco

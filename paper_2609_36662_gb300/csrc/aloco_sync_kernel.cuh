@@ -27,17 +27,56 @@ namespace aloco {
 // 128 (bf16) squared terms per fp32 partial.
 constexpr int kFlush = 16;
 
+// Tuning knobs (compile-time): packs loaded per thread before any is used,
+// minimum resident blocks per SM requested from the register allocator, and
+// the cache policy of the streaming loads and stores.
+#ifndef ALOCO_UNROLL
+#define ALOCO_UNROLL 1
+#endif
+#ifndef ALOCO_MINB
+#define ALOCO_MINB 0  // 0: the per-instance table below
+#endif
+#ifndef ALOCO_LD
+#define ALOCO_LD 0  // 0 ld.global.cs, 1 ld.global.lu, 2 plain, 3 ld.global.cg
+#endif
+#ifndef ALOCO_ST
+#define ALOCO_ST 0  // 0 st.global.cs, 1 plain, 2 st.global.cg
+#endif
+
+template <typename T>
+__device__ __forceinline__ T ld_stream(const T *p) {
+#if ALOCO_LD == 0
+    return __ldcs(p);
+#elif ALOCO_LD == 1
+    return __ldlu(p);
+#elif ALOCO_LD == 2
+    return *p;
+#else
+    return __ldcg(p);
+#endif
+}
+template <typename T>
+__device__ __forceinline__ void st_stream(T *p, T v) {
+#if ALOCO_ST == 0
+    __stcs(p, v);
+#elif ALOCO_ST == 1
+    *p = v;
+#else
+    __stcg(p, v);
+#endif
+}
+
 __device__ __forceinline__ float4 ldcs4(const void *base, int64_t i) {
-    return __ldcs(reinterpret_cast<const float4 *>(base) + i);
+    return ld_stream(reinterpret_cast<const float4 *>(base) + i);
 }
 __device__ __forceinline__ uint4 ldcs4u(const void *base, int64_t i) {
-    return __ldcs(reinterpret_cast<const uint4 *>(base) + i);
+    return ld_stream(reinterpret_cast<const uint4 *>(base) + i);
 }
 __device__ __forceinline__ void stcs4(void *base, int64_t i, float4 val) {
-    __stcs(reinterpret_cast<float4 *>(base) + i, val);
+    st_stream(reinterpret_cast<float4 *>(base) + i, val);
 }
 __device__ __forceinline__ void stcs4u(void *base, int64_t i, uint4 val) {
-    __stcs(reinterpret_cast<uint4 *>(base) + i, val);
+    st_stream(reinterpret_cast<uint4 *>(base) + i, val);
 }
 
 // Exact widening of the two bf16 values packed in a 32-bit word (element
@@ -74,8 +113,76 @@ __device__ __forceinline__ void outer_step(const Coef &k, float s, float g,
     gp = g + fmaf(k.ne_hi, d, k.ne_lo * d);
 }
 
+// One 16-byte replica access ("pack") and the matching theta / v elements.
+// fp32 replicas: 4 elements, one float4 of each stream.  bf16 replicas: 8
+// elements, one uint4 of each replica and two float4 of theta and v.
+template <bool BF16>
+struct Pack;
+
+template <>
+struct Pack<false> {
+    static constexpr int E = 4;
+    using Raw = float4;
+    __device__ static void load(const float *p, int64_t i, float (&o)[E]) {
+        const float4 t = ldcs4(p, i);
+        o[0] = t.x; o[1] = t.y; o[2] = t.z; o[3] = t.w;
+    }
+    __device__ static void store(float *p, int64_t i, const float (&o)[E]) {
+        stcs4(p, i, make_float4(o[0], o[1], o[2], o[3]));
+    }
+    __device__ static Raw load_x(const void *p, int64_t i) { return ldcs4(p, i); }
+    __device__ static void widen(const Raw &r, float (&o)[E]) {
+        o[0] = r.x; o[1] = r.y; o[2] = r.z; o[3] = r.w;
+    }
+    __device__ static Raw narrow(const float (&o)[E]) {
+        return make_float4(o[0], o[1], o[2], o[3]);
+    }
+    __device__ static void store_x(void *p, int64_t i, const Raw &r) {
+        stcs4(p, i, r);
+    }
+};
+
+template <>
+struct Pack<true> {
+    static constexpr int E = 8;
+    using Raw = uint4;
+    __device__ static void load(const float *p, int64_t i, float (&o)[E]) {
+        const float4 a = ldcs4(p, 2 * i), b = ldcs4(p, 2 * i + 1);
+        o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
+        o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
+    }
+    __device__ static void store(float *p, int64_t i, const float (&o)[E]) {
+        stcs4(p, 2 * i, make_float4(o[0], o[1], o[2], o[3]));
+        stcs4(p, 2 * i + 1, make_float4(o[4], o[5], o[6], o[7]));
+    }
+    __device__ static Raw load_x(const void *p, int64_t i) { return ldcs4u(p, i); }
+    __device__ static void widen(const Raw &r, float (&o)[E]) {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            o[2 * j] = bf16_lo(w[j]);
+            o[2 * j + 1] = bf16_hi(w[j]);
+        }
+    }
+    __device__ static Raw narrow(const float (&o)[E]) {
+        return make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]),
+                          pack_bf16x2(o[4], o[5]), pack_bf16x2(o[6], o[7]));
+    }
+    __device__ static void store_x(void *p, int64_t i, const Raw &r) {
+        stcs4u(p, i, r);
+    }
+};
+
+// Minimum resident blocks per SM the register allocator must allow (it
+// bounds registers per thread to 65536 / (kBlock * value)); 0 leaves the
+// choice to the compiler, which measured as good as any fixed budget.
 template <int MT, bool BF16>
-__global__ void __launch_bounds__(kBlock)
+constexpr int min_blocks() {
+    return ALOCO_MINB > 0 ? ALOCO_MINB : 0;
+}
+
+template <int MT, bool BF16>
+__global__ void __launch_bounds__(kBlock, (min_blocks<MT, BF16>()))
     sync_kernel(const __grid_constant__ SyncArgs a) {
     constexpr int MM = MT > 0 ? MT : ALOCO_MAX_WORKERS;
     const int M = MT > 0 ? MT : a.M;
@@ -107,92 +214,96 @@ __global__ void __launch_bounds__(kBlock)
     };
 
     // ---------------------------------------------------- vector body
-    if constexpr (!BF16) {
-        for (int64_t i = tid; i < a.nvec; i += stride) {
-            const float4 g4 = ldcs4(a.g, i);
-            const float4 v4 = ldcs4(a.v, i);
-            float s[4] = {0.f, 0.f, 0.f, 0.f};
-            const float gg[4] = {g4.x, g4.y, g4.z, g4.w};
+    using P = Pack<BF16>;
+    constexpr int E = P::E;
+
+    // Pseudo-gradients of one replica pack: S += Delta, ||Delta_m||^2 += Delta^2.
+    auto accumulate = [&](const float (&gg)[E], const typename P::Raw &raw,
+                          float (&s)[E], float &e) {
+        float xx[E];
+        P::widen(raw, xx);
 #pragma unroll
-            for (int m = 0; m < MM; ++m) {
-                if (MT == 0 && m >= M) continue;
-                const float4 x4 = ldcs4(a.x[m], i);
-                const float xx[4] = {x4.x, x4.y, x4.z, x4.w};
+        for (int j = 0; j < E; ++j) {
+            const float d = gg[j] - xx[j];
+            s[j] += d;
+            e = fmaf(d, d, e);
+        }
+    };
+    // Outer step of the pack and its stores: theta', v', replica reset.
+    auto finish = [&](int64_t i, const float (&gg)[E], const float (&vv)[E],
+                      const float (&s)[E]) {
+        float gp[E], vp[E];
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float d = gg[j] - xx[j];
-                    s[j] += d;
-                    e32[m] = fmaf(d, d, e32[m]);
-                }
+        for (int j = 0; j < E; ++j) {
+            b32 = fmaf(s[j], s[j], b32);
+            outer_step(k, s[j], gg[j], vv[j], gp[j], vp[j]);
+            nf += not_finite(gp[j], vp[j]);
+        }
+        P::store(a.g, i, gp);
+        P::store(a.v, i, vp);
+        const typename P::Raw xo = P::narrow(gp);
+#pragma unroll
+        for (int m = 0; m < MM; ++m) {
+            if (MT == 0 && m >= M) continue;
+            P::store_x(a.x[m], i, xo);
+        }
+        if (++cnt == kFlush) {
+            flush();
+            cnt = 0;
+        }
+    };
+
+    if constexpr (MT > 0) {
+        // Compile-time M: every load of the U packs is issued before any is
+        // used, so (M + 2) U 16-byte loads (bf16: (M + 4) U) are in flight.
+        constexpr int U = ALOCO_UNROLL;
+        for (int64_t i0 = tid; i0 < a.nvec; i0 += stride * U) {
+            float G[U][E], V[U][E];
+            typename P::Raw X[U][MT];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int64_t i = i0 + u * stride;
+                if (i >= a.nvec) continue;
+                P::load(a.g, i, G[u]);
+                P::load(a.v, i, V[u]);
+#pragma unroll
+                for (int m = 0; m < MT; ++m) X[u][m] = P::load_x(a.x[m], i);
             }
-            const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-            float gp[4], vp[4];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                b32 = fmaf(s[j], s[j], b32);
-                outer_step(k, s[j], gg[j], vv[j], gp[j], vp[j]);
-                nf += not_finite(gp[j], vp[j]);
-            }
-            const float4 go = make_float4(gp[0], gp[1], gp[2], gp[3]);
-            stcs4(a.g, i, go);
-            stcs4(a.v, i, make_float4(vp[0], vp[1], vp[2], vp[3]));
+            for (int u = 0; u < U; ++u) {
+                const int64_t i = i0 + u * stride;
+                if (i >= a.nvec) continue;
+                float s[E];
 #pragma unroll
-            for (int m = 0; m < MM; ++m) {
-                if (MT == 0 && m >= M) continue;
-                stcs4(a.x[m], i, go);
-            }
-            if (++cnt == kFlush) {
-                flush();
-                cnt = 0;
+                for (int j = 0; j < E; ++j) s[j] = 0.f;
+#pragma unroll
+                for (int m = 0; m < MT; ++m) accumulate(G[u], X[u][m], s, e32[m]);
+                finish(i, G[u], V[u], s);
             }
         }
     } else {
+        // Any M up to 32: replicas are loaded in groups of 8 (independent
+        // loads in flight) and consumed group by group, which bounds the
+        // registers that hold loaded packs.
+        constexpr int kGroup = 8;
         for (int64_t i = tid; i < a.nvec; i += stride) {
-            const float4 g4a = ldcs4(a.g, 2 * i), g4b = ldcs4(a.g, 2 * i + 1);
-            const float4 v4a = ldcs4(a.v, 2 * i), v4b = ldcs4(a.v, 2 * i + 1);
-            const float gg[8] = {g4a.x, g4a.y, g4a.z, g4a.w,
-                                 g4b.x, g4b.y, g4b.z, g4b.w};
-            float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            float gg[E], vv[E], s[E];
+            P::load(a.g, i, gg);
+            P::load(a.v, i, vv);
 #pragma unroll
-            for (int m = 0; m < MM; ++m) {
-                if (MT == 0 && m >= M) continue;
-                const uint4 x4 = ldcs4u(a.x[m], i);
-                const uint32_t w[4] = {x4.x, x4.y, x4.z, x4.w};
+            for (int j = 0; j < E; ++j) s[j] = 0.f;
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float d0 = gg[2 * j] - bf16_lo(w[j]);
-                    const float d1 = gg[2 * j + 1] - bf16_hi(w[j]);
-                    s[2 * j] += d0;
-                    s[2 * j + 1] += d1;
-                    e32[m] = fmaf(d0, d0, e32[m]);
-                    e32[m] = fmaf(d1, d1, e32[m]);
-                }
-            }
-            const float vv[8] = {v4a.x, v4a.y, v4a.z, v4a.w,
-                                 v4b.x, v4b.y, v4b.z, v4b.w};
-            float gp[8], vp[8];
+            for (int m0 = 0; m0 < MM; m0 += kGroup) {
+                if (m0 >= M) break;
+                typename P::Raw X[kGroup];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                b32 = fmaf(s[j], s[j], b32);
-                outer_step(k, s[j], gg[j], vv[j], gp[j], vp[j]);
-                nf += not_finite(gp[j], vp[j]);
-            }
-            stcs4(a.g, 2 * i, make_float4(gp[0], gp[1], gp[2], gp[3]));
-            stcs4(a.g, 2 * i + 1, make_float4(gp[4], gp[5], gp[6], gp[7]));
-            stcs4(a.v, 2 * i, make_float4(vp[0], vp[1], vp[2], vp[3]));
-            stcs4(a.v, 2 * i + 1, make_float4(vp[4], vp[5], vp[6], vp[7]));
-            const uint4 xo = make_uint4(
-                pack_bf16x2(gp[0], gp[1]), pack_bf16x2(gp[2], gp[3]),
-                pack_bf16x2(gp[4], gp[5]), pack_bf16x2(gp[6], gp[7]));
+                for (int q = 0; q < kGroup; ++q)
+                    if (m0 + q < M) X[q] = P::load_x(a.x[m0 + q], i);
 #pragma unroll
-            for (int m = 0; m < MM; ++m) {
-                if (MT == 0 && m >= M) continue;
-                stcs4u(a.x[m], i, xo);
+                for (int q = 0; q < kGroup; ++q)
+                    if (m0 + q < M) accumulate(gg, X[q], s, e32[m0 + q]);
             }
-            if (++cnt == kFlush) {
-                flush();
-                cnt = 0;
-            }
+            finish(i, gg, vv, s);
         }
     }
 
@@ -327,19 +438,32 @@ __global__ void __launch_bounds__(kBlock)
     }
 }
 
-// Occupancy-sized persistent grid for one instance.
+// Tuned residency (blocks of kBlock threads per SM) of the fused pass for
+// M workers, measured on GB300 over M = 1..32 and both replica types on a
+// 2^28-parameter round: fewer resident warps streaming more arrays keep
+// HBM busier once M + 2 streams are in flight.  Capped by occupancy.
+template <bool BF16>
+constexpr int tuned_blocks_per_sm(int M) {
+    if (BF16) return M <= 7 ? 2 : 1;
+    return M == 1 ? 4 : M == 2 ? 3 : M <= 8 ? 2 : 1;
+}
+
+// Persistent grid for one instance: SMs x resident blocks.
 template <int MT, bool BF16>
-cudaError_t plan_one(int64_t work_items, int sm_count, LaunchPlan *plan) {
-    static int blocks_per_sm = 0;  // per instance, computed once
+cudaError_t plan_one(int64_t work_items, int sm_count, int M, int request,
+                     LaunchPlan *plan) {
+    static int occupancy = 0;  // per instance, computed once
     const void *fn = reinterpret_cast<const void *>(&sync_kernel<MT, BF16>);
-    if (blocks_per_sm == 0) {
+    if (occupancy == 0) {
         int b = 0;
         cudaError_t e =
             cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, sync_kernel<MT, BF16>,
                                                           kBlock, 0);
         if (e != cudaSuccess) return e;
-        blocks_per_sm = b > 0 ? b : 1;
+        occupancy = b > 0 ? b : 1;
     }
+    int blocks_per_sm = request > 0 ? request : tuned_blocks_per_sm<BF16>(M);
+    if (blocks_per_sm <= 0 || blocks_per_sm > occupancy) blocks_per_sm = occupancy;
     int64_t want = (work_items + kBlock - 1) / kBlock;
     int64_t full = (int64_t)sm_count * blocks_per_sm;
     int64_t grid = want < full ? want : full;
@@ -352,18 +476,19 @@ cudaError_t plan_one(int64_t work_items, int sm_count, LaunchPlan *plan) {
 
 template <bool BF16>
 cudaError_t plan_dispatch(int M, int64_t work_items, int sm_count,
-                          LaunchPlan *plan) {
+                          int blocks_per_sm, LaunchPlan *plan) {
     switch (M) {
 #define ALOCO_CASE(K) \
     case K:           \
-        return plan_one<K, BF16>(work_items, sm_count, plan);
+        return plan_one<K, BF16>(work_items, sm_count, M, blocks_per_sm, plan);
         ALOCO_CASE(1) ALOCO_CASE(2) ALOCO_CASE(3) ALOCO_CASE(4)
         ALOCO_CASE(5) ALOCO_CASE(6) ALOCO_CASE(7) ALOCO_CASE(8)
         ALOCO_CASE(9) ALOCO_CASE(10) ALOCO_CASE(11) ALOCO_CASE(12)
         ALOCO_CASE(13) ALOCO_CASE(14) ALOCO_CASE(15) ALOCO_CASE(16)
 #undef ALOCO_CASE
         default:
-            return plan_one<0, BF16>(work_items, sm_count, plan);
+            return plan_one<0, BF16>(work_items, sm_count, M, blocks_per_sm,
+                                     plan);
     }
 }
 
