@@ -42,7 +42,7 @@ METRIC = ("outer-sync rounds/s and achieved HBM GB/s (fraction of GB300 "
 UNIT = "rounds/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-KERNEL_NAME = "sync_kernel"
+PASSES = {"auto": 0, "registers": 1, "bulk_copy": 2}
 
 
 def workloads_by_name():
@@ -87,7 +87,7 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload: str):
+def recorded_traffic(workload: str, kernel: str):
     """DRAM bytes per launch of the fused pass from the committed ncu
     summary, if it was taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
@@ -96,7 +96,7 @@ def recorded_traffic(workload: str):
             rec = json.load(f)
     except Exception:
         return None
-    entry = rec.get(workload)
+    entry = rec.get(f"{workload}/{kernel}")
     if not entry or entry.get("kernel_hash") != kernel_source_hash():
         return None
     return entry.get("dram_bytes_per_launch")
@@ -328,7 +328,7 @@ def run_cuda(args, w):
                                   f"{w.M} workers of one round "
                                   f"({t:.1f} s), scaled to a full round"}
 
-    opts = A.default_opts(time_kernel=1)
+    opts = A.default_opts(time_kernel=1, pass_=PASSES[args.pass_])
     step_ms, kern_ms, statuses = [], [], []
     ev = [(torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in rounds]
@@ -352,9 +352,11 @@ def run_cuda(args, w):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     t_wall = time.perf_counter()
+    st_first = None
     with ClockSampler(device.index) as clocks:
         for k in range(args.warmup, args.warmup + args.steps):
             st = one_round(k)
+            st_first = st_first or st
             statuses.append(st["status"])
             kern_ms.append(st["kernel_ms"])
         torch.cuda.synchronize()
@@ -365,6 +367,8 @@ def run_cuda(args, w):
     for k in range(args.warmup, args.warmup + args.steps):
         step_ms.append(ev[k][0].elapsed_time(ev[k][1]))
 
+    kernel_name = ("sync_tma_kernel" if st_first.get("pass_used") == 2
+                   else "sync_kernel")
     ms_step = statistics.mean(step_ms)
     ms_step = reduce_max(ms_step, world, device)
     ms_kern = reduce_max(statistics.mean(kern_ms), world, device)
@@ -395,8 +399,8 @@ def run_cuda(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
                          "unit": "GB/s", "frac": achieved / peak,
                          "peak_source": peak_kind,
-                         "traffic": recorded_traffic(w.name),
-                         "kernel": KERNEL_NAME,
+                         "traffic": recorded_traffic(w.name, kernel_name),
+                         "kernel": kernel_name,
                          "algorithmic_bytes_per_launch": w.bytes_per_round()},
             "cpu_baseline": cpu_baseline,
             "e2e": e2e,
@@ -480,6 +484,8 @@ def main(argv=None):
     p.add_argument("--e2e-warmup", type=int, default=2)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--pass", dest="pass_", choices=sorted(PASSES),
+                   default="auto", help="which fused kernel runs the round")
     p.add_argument("--list", action="store_true")
     args = p.parse_args(argv)
     table = workloads_by_name()

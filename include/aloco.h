@@ -105,10 +105,26 @@ typedef enum {
     ALOCO_CORR_NONE = 2
 } aloco_corr_mode;
 
+/* The two implementations of the fused pass.  Both compute the same round
+ * with the same arithmetic; they differ in how data reaches the SMs.
+ *   REGISTERS  every thread streams 16-byte loads of theta, v and the
+ *              replicas straight into registers (any M, any alignment);
+ *   BULK_COPY  a producer warp per SM stages 4-8 KB tiles of every array in
+ *              a shared-memory ring with cp.async.bulk and mbarriers, and
+ *              consumer warps compute from shared memory (M <= 16, 16-byte
+ *              aligned buffers; otherwise REGISTERS runs);
+ *   AUTO       the faster of the two as measured on GB300: at present the
+ *              register-streaming pass for every (M, dtype). */
+typedef enum {
+    ALOCO_PASS_AUTO = 0,
+    ALOCO_PASS_REGISTERS = 1,
+    ALOCO_PASS_BULK_COPY = 2
+} aloco_pass;
+
 /* Options.  aloco_default_opts() fills the paper's settings
  * (Tab. AutoLoCo configuration): mu_min 0.45, mu_max 0.90, kappa_max 1.6,
  * eps 1e-8, normalize off, FULL correction, no kernel timing, the tuned
- * launch configuration, default stream.  Passing NULL where an opts pointer is accepted means these
+ * launch configuration, default stream, AUTO pass.  Passing NULL where an opts pointer is accepted means these
  * defaults. */
 typedef struct aloco_opts {
     double mu_min;
@@ -126,6 +142,8 @@ typedef struct aloco_opts {
                              sums, so a different value can change the
                              statistics in their last bits.                  */
     void *stream;         /* cudaStream_t; NULL = legacy default stream      */
+    int32_t pass;         /* aloco_pass: which fused kernel runs the round   */
+    int32_t reserved;
 } aloco_opts_t;
 
 /* Correction context of one interval (App. B.2, B.4). */
@@ -152,7 +170,7 @@ typedef struct aloco_stats {
     int32_t M;
     int32_t grid;                     /* CUDA blocks of the fused pass       */
     float kernel_ms;                  /* fused-pass duration, or -1          */
-    int32_t reserved;
+    int32_t pass_used;                /* aloco_pass that ran (0 if no kernel) */
 } aloco_stats_t;
 
 /* Fill *opts with the defaults listed above. */

@@ -16,6 +16,7 @@ MAX_WORKERS = 32
 F32, BF16 = 0, 1
 SCHED_COSINE, SCHED_CONSTANT, SCHED_LINEAR = 0, 1, 2
 CORR_FULL, CORR_MOMENTUM_ONLY, CORR_NONE = 0, 1, 2
+PASS_AUTO, PASS_REGISTERS, PASS_BULK_COPY = 0, 1, 2
 
 OK = 0
 ERR_ARG = -1
@@ -51,7 +52,8 @@ class Opts(ctypes.Structure):
                 ("normalize", ctypes.c_int32), ("mode", ctypes.c_int32),
                 ("time_kernel", ctypes.c_int32),
                 ("blocks_per_sm", ctypes.c_int32),
-                ("stream", ctypes.c_void_p)]
+                ("stream", ctypes.c_void_p), ("pass_", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
 
 
 class Correction(ctypes.Structure):
@@ -69,13 +71,14 @@ class Stats(ctypes.Structure):
                 ("drift", ctypes.c_double * MAX_WORKERS),
                 ("corr", Correction), ("nonfinite", ctypes.c_int64),
                 ("M", ctypes.c_int32), ("grid", ctypes.c_int32),
-                ("kernel_ms", ctypes.c_float), ("reserved", ctypes.c_int32)]
+                ("kernel_ms", ctypes.c_float), ("pass_used", ctypes.c_int32)]
 
     def as_dict(self):
         return {"D": self.D, "C": self.C, "mean_sq_norm": self.mean_sq_norm,
                 "drift": list(self.drift[:self.M]),
                 "corr": self.corr.as_dict(), "nonfinite": self.nonfinite,
-                "M": self.M, "grid": self.grid, "kernel_ms": self.kernel_ms}
+                "M": self.M, "grid": self.grid, "kernel_ms": self.kernel_ms,
+                "pass_used": self.pass_used}
 
 
 class AlocoError(RuntimeError):

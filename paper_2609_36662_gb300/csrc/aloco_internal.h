@@ -34,7 +34,22 @@ struct SyncArgs {
     unsigned int *ticket;           // last-block-done counter, 0 between launches
     double *totals;                 // [M + 1] fixed-order totals
     unsigned long long *nf_total;   // [1]
+    // bulk-copy pass only
+    int64_t n_tiles;                // whole tiles of kTmaConsumers packs
+    int stages;                     // depth of the shared-memory ring
+    unsigned int *error;            // set to 1 if a pipeline wait timed out
 };
+
+// Slots of the totals block read back after a round (8 bytes each): M + 1
+// totals, then the non-finite count, then the pipeline error word.
+constexpr int kTotalsSlots = ALOCO_MAX_WORKERS + 3;
+constexpr int kNfSlot = ALOCO_MAX_WORKERS + 1;
+constexpr int kErrorSlot = ALOCO_MAX_WORKERS + 2;
+
+// Shared memory the bulk-copy pass may use for its ring (bytes), and the
+// packs of one tile (one per consumer thread).
+constexpr int kTmaSmemBudget = 224 * 1024;
+constexpr int kTmaTilePacks = 256;
 
 // Elements per vector pack: one 16-byte access of a replica.
 inline int pack_elems(aloco_dtype dt) { return dt == ALOCO_F32 ? 4 : 8; }
@@ -44,6 +59,9 @@ struct LaunchPlan {
     const void *kernel;
     int grid;
     int block;
+    int smem = 0;       // dynamic shared memory (bytes)
+    int stages = 0;     // bulk-copy pass: ring depth
+    int64_t tiles = 0;  // bulk-copy pass: whole tiles
 };
 
 // Pick the kernel instance and grid; returns cudaSuccess or an error.
@@ -53,6 +71,16 @@ cudaError_t plan_sync_f32(int M, int64_t work_items, int sm_count,
                           int blocks_per_sm, LaunchPlan *plan);
 cudaError_t plan_sync_bf16(int M, int64_t work_items, int sm_count,
                            int blocks_per_sm, LaunchPlan *plan);
+
+// The bulk-copy (TMA) pass for 1 <= M <= 16 and 16-byte aligned buffers.
+cudaError_t plan_sync_tma_f32(int M, int64_t nvec, int sm_count,
+                              LaunchPlan *plan);
+cudaError_t plan_sync_tma_bf16(int M, int64_t nvec, int sm_count,
+                               LaunchPlan *plan);
+
+// Whether a round of M workers (dtype) uses the bulk-copy pass, given the
+// requested aloco_pass.
+bool use_tma(int pass, int M, aloco_dtype dtype, int64_t nvec);
 
 // Host helpers shared by the entry points (aloco_host.cpp).
 int report_error(int code, const char *msg);

@@ -34,7 +34,7 @@ constexpr int kScratchBlocks = ALOCO_NOALLOC_MAX_BLOCKS;
 struct NoallocScratch {
     double partials[kScratchBlocks * (ALOCO_MAX_WORKERS + 1)];
     unsigned long long nf_partials[kScratchBlocks];
-    double totals[ALOCO_MAX_WORKERS + 2];  // M + 1 totals, then the nf count
+    double totals[aloco::kTotalsSlots];  // M + 1 totals, nf count, error word
     unsigned int ticket;
 };
 
@@ -176,9 +176,15 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
 
     const int64_t work = a.nvec > 0 ? a.nvec : a.n;
     aloco::LaunchPlan plan;
-    e = dtype == ALOCO_F32
-            ? aloco::plan_sync_f32(M, work, g_sms[device], o.blocks_per_sm, &plan)
-            : aloco::plan_sync_bf16(M, work, g_sms[device], o.blocks_per_sm, &plan);
+    const bool tma = aloco::use_tma(o.pass, M, dtype, a.nvec);
+    if (tma)
+        e = dtype == ALOCO_F32
+                ? aloco::plan_sync_tma_f32(M, a.nvec, g_sms[device], &plan)
+                : aloco::plan_sync_tma_bf16(M, a.nvec, g_sms[device], &plan);
+    else
+        e = dtype == ALOCO_F32
+                ? aloco::plan_sync_f32(M, work, g_sms[device], o.blocks_per_sm, &plan)
+                : aloco::plan_sync_bf16(M, work, g_sms[device], o.blocks_per_sm, &plan);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return errf(ALOCO_ERR_CUDA, "launch plan: %s", cudaGetErrorString(e));
@@ -194,24 +200,29 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
     a.nf_partials = s->nf_partials;
     a.ticket = &s->ticket;
     a.totals = s->totals;
-    a.nf_total = (unsigned long long *)(s->totals + ALOCO_MAX_WORKERS + 1);
+    a.nf_total = (unsigned long long *)(s->totals + aloco::kNfSlot);
+    a.error = (unsigned int *)(s->totals + aloco::kErrorSlot);
+    a.n_tiles = plan.tiles;
+    a.stages = plan.stages;
 
     cudaStream_t stream = (cudaStream_t)o.stream;
-    // The ticket must start at zero; every partial row and total used by
-    // this launch is written by it before it is read.
+    // The ticket and the error word must start at zero; every partial row
+    // and total used by this launch is written by it before it is read.
     e = cudaMemsetAsync(&s->ticket, 0, sizeof(unsigned int), stream);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(a.error, 0, sizeof(unsigned int), stream);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return errf(ALOCO_ERR_CUDA, "ticket reset: %s", cudaGetErrorString(e));
     }
     void *params[] = {&a};
     e = cudaLaunchKernel(plan.kernel, dim3(plan.grid), dim3(plan.block), params,
-                         0, stream);
+                         plan.smem, stream);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return errf(ALOCO_ERR_CUDA, "fused sync launch: %s", cudaGetErrorString(e));
     }
-    double host[ALOCO_MAX_WORKERS + 2];
+    double host[aloco::kTotalsSlots];
     e = cudaMemcpyAsync(host, s->totals, sizeof host, cudaMemcpyDeviceToHost,
                         stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
@@ -220,9 +231,15 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
         return errf(ALOCO_ERR_CUDA, "round: %s", cudaGetErrorString(e));
     }
     unsigned long long nf;
-    std::memcpy(&nf, host + ALOCO_MAX_WORKERS + 1, sizeof nf);
+    std::memcpy(&nf, host + aloco::kNfSlot, sizeof nf);
+    unsigned int perr;
+    std::memcpy(&perr, host + aloco::kErrorSlot, sizeof perr);
+    if (perr != 0)
+        return errf(ALOCO_ERR_CUDA,
+                    "bulk-copy pipeline wait timed out; outputs are incomplete");
     aloco::finalize_stats(host, nf, M, o.eps, st);
     st->grid = plan.grid;
+    st->pass_used = tma ? ALOCO_PASS_BULK_COPY : ALOCO_PASS_REGISTERS;
     if (st->nonfinite > 0 || !std::isfinite(st->D) || !std::isfinite(st->C))
         return errf(ALOCO_ERR_NONFINITE,
                     "round produced %lld non-finite elements (D=%g, C=%g)",

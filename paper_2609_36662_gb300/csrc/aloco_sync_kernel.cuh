@@ -173,6 +173,102 @@ struct Pack<true> {
     }
 };
 
+// Block and grid reduction of the per-thread fp64 partials (the block's
+// NW warps all call it).  Each block writes one row of M + 1 partials; the
+// last block to finish (atomic ticket, no spinning) adds the rows in block
+// order and resets the ticket.  The order of every addition is fixed by the
+// grid alone.
+template <int MM, int NW>
+__device__ __forceinline__ void reduce_and_finish(const SyncArgs &a, int M,
+                                                  double (&e64)[MM], double b64,
+                                                  unsigned nf) {
+    constexpr int kThreads = NW * 32;
+    __shared__ double sh[NW][MM + 1];
+    __shared__ unsigned long long shnf[NW];
+    __shared__ bool s_last;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+    unsigned long long nfl = nf;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+#pragma unroll
+        for (int m = 0; m < MM; ++m)
+            e64[m] += __shfl_down_sync(0xffffffffu, e64[m], off);
+        b64 += __shfl_down_sync(0xffffffffu, b64, off);
+        nfl += __shfl_down_sync(0xffffffffu, nfl, off);
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int m = 0; m < MM; ++m) sh[warp][m] = e64[m];
+        sh[warp][MM] = b64;
+        shnf[warp] = nfl;
+    }
+    __syncthreads();
+    const int np = M + 1;  // values per block: M energies + sum S^2
+    if (threadIdx.x < np) {
+        const int col = threadIdx.x < M ? threadIdx.x : MM;
+        double t = 0.0;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) t += sh[w][col];
+        a.partials[(int64_t)blockIdx.x * np + threadIdx.x] = t;
+    }
+    if (threadIdx.x == kThreads - 1) {
+        unsigned long long t = 0;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) t += shnf[w];
+        a.nf_partials[blockIdx.x] = t;
+    }
+
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const unsigned prev = atomicAdd(a.ticket, 1u);
+        s_last = (prev == gridDim.x - 1);
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+
+    double acc[MM + 1];
+#pragma unroll
+    for (int p = 0; p <= MM; ++p) acc[p] = 0.0;
+    unsigned long long nacc = 0;
+    for (int b = threadIdx.x; b < (int)gridDim.x; b += kThreads) {
+        const double *row = a.partials + (int64_t)b * np;
+#pragma unroll
+        for (int p = 0; p <= MM; ++p)
+            if (p < np) acc[p] += __ldcg(row + p);
+        nacc += __ldcg(a.nf_partials + b);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+#pragma unroll
+        for (int p = 0; p <= MM; ++p)
+            acc[p] += __shfl_down_sync(0xffffffffu, acc[p], off);
+        nacc += __shfl_down_sync(0xffffffffu, nacc, off);
+    }
+    __syncthreads();  // sh is reused
+    if (lane == 0) {
+#pragma unroll
+        for (int p = 0; p <= MM; ++p) sh[warp][p] = acc[p];
+        shnf[warp] = nacc;
+    }
+    __syncthreads();
+    if (threadIdx.x < np) {
+        double t = 0.0;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) t += sh[w][threadIdx.x];
+        a.totals[threadIdx.x] = t;
+    }
+    if (threadIdx.x == kThreads - 1) {
+        unsigned long long t = 0;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) t += shnf[w];
+        *a.nf_total = t;
+        *a.ticket = 0u;  // ready for the next launch
+    }
+}
+
 // Minimum resident blocks per SM the register allocator must allow (it
 // bounds registers per thread to 65536 / (kBlock * value)); 0 leaves the
 // choice to the compiler, which measured as good as any fixed budget.
@@ -349,93 +445,7 @@ __global__ void __launch_bounds__(kBlock, (min_blocks<MT, BF16>()))
     }
     flush();
 
-    // ------------------------------------------------ block reduction
-    constexpr int kWarps = kBlock / 32;
-    __shared__ double sh[kWarps][MM + 1];
-    __shared__ unsigned long long shnf[kWarps];
-    __shared__ bool s_last;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-
-    unsigned long long nfl = nf;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-#pragma unroll
-        for (int m = 0; m < MM; ++m)
-            e64[m] += __shfl_down_sync(0xffffffffu, e64[m], off);
-        b64 += __shfl_down_sync(0xffffffffu, b64, off);
-        nfl += __shfl_down_sync(0xffffffffu, nfl, off);
-    }
-    if (lane == 0) {
-#pragma unroll
-        for (int m = 0; m < MM; ++m) sh[warp][m] = e64[m];
-        sh[warp][MM] = b64;
-        shnf[warp] = nfl;
-    }
-    __syncthreads();
-    const int np = M + 1;  // values per block: M energies + sum S^2
-    if (threadIdx.x < np) {
-        const int col = threadIdx.x < M ? threadIdx.x : MM;
-        double t = 0.0;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) t += sh[w][col];
-        a.partials[(int64_t)blockIdx.x * np + threadIdx.x] = t;
-    }
-    if (threadIdx.x == kBlock - 1) {
-        unsigned long long t = 0;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) t += shnf[w];
-        a.nf_partials[blockIdx.x] = t;
-    }
-
-    // ------------------------------------------- last block: grid total
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        const unsigned prev = atomicAdd(a.ticket, 1u);
-        s_last = (prev == gridDim.x - 1);
-    }
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-
-    double acc[MM + 1];
-#pragma unroll
-    for (int p = 0; p <= MM; ++p) acc[p] = 0.0;
-    unsigned long long nacc = 0;
-    for (int b = threadIdx.x; b < (int)gridDim.x; b += kBlock) {
-        const double *row = a.partials + (int64_t)b * np;
-#pragma unroll
-        for (int p = 0; p <= MM; ++p)
-            if (p < np) acc[p] += __ldcg(row + p);
-        nacc += __ldcg(a.nf_partials + b);
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-#pragma unroll
-        for (int p = 0; p <= MM; ++p)
-            acc[p] += __shfl_down_sync(0xffffffffu, acc[p], off);
-        nacc += __shfl_down_sync(0xffffffffu, nacc, off);
-    }
-    __syncthreads();  // sh is reused
-    if (lane == 0) {
-#pragma unroll
-        for (int p = 0; p <= MM; ++p) sh[warp][p] = acc[p];
-        shnf[warp] = nacc;
-    }
-    __syncthreads();
-    if (threadIdx.x < np) {
-        double t = 0.0;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) t += sh[w][threadIdx.x];
-        a.totals[threadIdx.x] = t;
-    }
-    if (threadIdx.x == kBlock - 1) {
-        unsigned long long t = 0;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) t += shnf[w];
-        *a.nf_total = t;
-        *a.ticket = 0u;  // ready for the next launch
-    }
+    reduce_and_finish<MM, kBlock / 32>(a, M, e64, b64, nf);
 }
 
 // Tuned residency (blocks of kBlock threads per SM) of the fused pass for

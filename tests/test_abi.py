@@ -56,7 +56,7 @@ def test_struct_layout_matches_c(tmp_path):
 int main(void) {
   printf("%zu %zu %zu %zu\n", sizeof(aloco_schedule_t), sizeof(aloco_opts_t),
          sizeof(aloco_correction_t), sizeof(aloco_stats_t));
-  printf("%zu %zu %zu %zu %zu %zu\n", offsetof(aloco_opts_t, stream),
+  printf("%zu %zu %zu %zu %zu %zu %zu\n", offsetof(aloco_opts_t, pass), offsetof(aloco_opts_t, stream),
          offsetof(aloco_stats_t, corr), offsetof(aloco_stats_t, nonfinite),
          offsetof(aloco_stats_t, kernel_ms), offsetof(aloco_schedule_t, peak_lr),
          offsetof(aloco_schedule_t, total_steps));
@@ -72,7 +72,8 @@ int main(void) {
     offs = list(map(int, lines[1].split()))
     assert sizes == [ctypes.sizeof(A.Schedule), ctypes.sizeof(A.Opts),
                      ctypes.sizeof(A.Correction), ctypes.sizeof(A.Stats)]
-    assert offs == [A.Opts.stream.offset, A.Stats.corr.offset,
+    assert offs == [A.Opts.pass_.offset, A.Opts.stream.offset,
+                    A.Stats.corr.offset,
                     A.Stats.nonfinite.offset, A.Stats.kernel_ms.offset,
                     A.Schedule.peak_lr.offset, A.Schedule.total_steps.offset]
 
@@ -84,6 +85,7 @@ def test_default_opts_are_the_papers_settings(lib):
     assert (o.mu_min, o.mu_max, o.kappa_max) == (0.45, 0.90, 1.6)
     assert o.eps == 1e-8 and o.normalize == 0 and o.mode == A.CORR_FULL
     assert o.stream is None and o.time_kernel == 0
+    assert o.pass_ == A.PASS_AUTO and o.blocks_per_sm == 0
 
 
 @pytest.mark.parametrize("kind", [0, 1, 2])
@@ -140,7 +142,9 @@ def test_correction_argument_errors(lib):
              dict(opts=A.default_opts(eps=0.0)),
              dict(opts=A.default_opts(mu_min=0.9, mu_max=0.5)),
              dict(opts=A.default_opts(kappa_max=0.5)),
-             dict(opts=A.default_opts(mode=9))]
+             dict(opts=A.default_opts(mode=9)),
+             dict(opts=A.default_opts(pass_=7)),
+             dict(opts=A.default_opts(blocks_per_sm=-1))]
     for kw in cases:
         args = dict(schedule=s, step=4000, H_sel=150, H_base=100,
                     outer_lr=0.7, outer_beta=0.9, opts=None)

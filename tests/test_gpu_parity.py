@@ -70,14 +70,25 @@ MEDIUM = [(1_000_003, m, dt) for m in (1, 3, 4, 8, 16, 17, 32)
           for dt in ("f32", "bf16")]
 
 
+PASSES = [A.PASS_REGISTERS, A.PASS_BULK_COPY]
+PASS_IDS = ["registers", "bulk_copy"]
+
+
+@pytest.mark.parametrize("pass_", PASSES, ids=PASS_IDS)
 @pytest.mark.parametrize("N,M,dt", SMALL + MEDIUM)
-def test_round_matches_oracle(N, M, dt):
+def test_round_matches_oracle(N, M, dt, pass_):
+    """Both fused passes against the oracle.  The bulk-copy pass serves M <=
+    16 with 16-byte aligned buffers and at least one whole tile; other
+    rounds fall back to the register-streaming pass."""
     w = W.small(N, M, dt, seed=N % 97 + M)
     g, v, xs = gpu_inputs(w)
     v.normal_(0, 1e-3)          # carried momentum
     orc = run_oracle_round(g, v, xs, w, w.start_step, w.H_sel[0])
-    st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0])
+    st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0],
+                       opts=A.default_opts(pass_=pass_))
     assert st["status"] == A.OK
+    tma_ok = M <= 16 and N * (4 if dt == "f32" else 2) >= 256 * 16
+    assert st["pass_used"] == (pass_ if tma_ok else A.PASS_REGISTERS)
     compare_round(w, st, orc, g, v, xs)
 
 
@@ -135,13 +146,15 @@ def test_direct_averaging_gives_the_mean_of_endpoints():
     assert_field(g.cpu().numpy(), mean.cpu().numpy(), "mean")
 
 
-def test_repeated_rounds_are_bit_identical():
+@pytest.mark.parametrize("pass_", PASSES, ids=PASS_IDS)
+def test_repeated_rounds_are_bit_identical(pass_):
     w = W.small(2_000_003, 8, "bf16", seed=5)
     results = []
     for _ in range(5):
         g, v, xs = gpu_inputs(w)
         v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(1))
-        st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0])
+        st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0],
+                           opts=A.default_opts(pass_=pass_))
         results.append((st["D"], st["C"], tuple(st["drift"]),
                         st["mean_sq_norm"], g.cpu().numpy().tobytes(),
                         v.cpu().numpy().tobytes(),
@@ -149,10 +162,12 @@ def test_repeated_rounds_are_bit_identical():
     assert all(r == results[0] for r in results[1:])
 
 
+@pytest.mark.parametrize("pass_", PASSES, ids=PASS_IDS)
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
-def test_guard_bands_untouched(dt):
+def test_guard_bands_untouched(dt, pass_):
     """Only [0, N) of each buffer is written: 64 sentinel elements on both
-    sides of every buffer stay intact."""
+    sides of every buffer stay intact.  (pad is 64 elements, so for fp32 the
+    buffers stay 16-byte aligned and the bulk-copy pass runs.)"""
     N, M, pad = 123_457, 3, 64
     w = W.small(N, M, dt, seed=9)
     g, v, xs = gpu_inputs(w)
@@ -164,7 +179,7 @@ def test_guard_bands_untouched(dt):
     xb = [padded(x, 3.0) for x in xs]
     st = run_gpu_round(gb[pad:pad + N], vb[pad:pad + N],
                        [x[pad:pad + N] for x in xb], w, w.start_step,
-                       w.H_sel[0])
+                       w.H_sel[0], opts=A.default_opts(pass_=pass_))
     assert st["status"] == A.OK
     for t, fill in [(gb, 7.0), (vb, -7.0)] + [(x, 3.0) for x in xb]:
         assert torch.all(t[:pad] == fill) and torch.all(t[-pad:] == fill)

@@ -40,11 +40,14 @@ def _round(w, g, v, xs, noalloc, opts=None):
                   outer_beta=w.outer_beta, opts=opts, noalloc=noalloc)
 
 
+@pytest.mark.parametrize("pass_", [A.PASS_AUTO, A.PASS_BULK_COPY],
+                         ids=["auto", "bulk_copy"])
 @pytest.mark.parametrize("dt,N,M", [("f32", 1_000_003, 8),
                                     ("bf16", 2_000_005, 5),
                                     ("f32", 4099, 17)])
-def test_noalloc_matches_the_allocating_entry_point(dt, N, M):
+def test_noalloc_matches_the_allocating_entry_point(dt, N, M, pass_):
     w = W.small(N, M, dt, seed=31)
+    opts = A.default_opts(pass_=pass_)
     for call in range(2):
         g, v, xs = gpu_inputs(w, round_index=call)
         v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(call))
@@ -52,11 +55,11 @@ def test_noalloc_matches_the_allocating_entry_point(dt, N, M):
         # the first call starts with the allocation-free entry point, so a
         # fresh process exercises its set-up before anything else
         if call == 0:
-            st_new = _round(w, g2, v2, xs2, noalloc=True)
-            st_ref = _round(w, g, v, xs, noalloc=False)
+            st_new = _round(w, g2, v2, xs2, noalloc=True, opts=opts)
+            st_ref = _round(w, g, v, xs, noalloc=False, opts=opts)
         else:
-            st_ref = _round(w, g, v, xs, noalloc=False)
-            st_new = _round(w, g2, v2, xs2, noalloc=True)
+            st_ref = _round(w, g, v, xs, noalloc=False, opts=opts)
+            st_new = _round(w, g2, v2, xs2, noalloc=True, opts=opts)
         assert st_new["status"] == A.OK and st_ref["status"] == A.OK
         assert st_new["kernel_ms"] == -1.0
         assert st_new["nonfinite"] == st_ref["nonfinite"] == 0
