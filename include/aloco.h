@@ -233,6 +233,171 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
                   double outer_beta, const aloco_opts_t *opts,
                   aloco_stats_t *stats_out);
 
+/* ------------------------------------------------------------------------
+ * Interval controller (Sec. 3.1; App. A).  Host-only and scalar: after each
+ * completed interval it takes that interval's D_t, C_t, accumulated inner
+ * learning rate and token count, assesses them against the accepted-horizon
+ * reference profile and returns the horizon of the next interval, in tokens
+ * and in executable steps, together with the step horizon of one base token
+ * interval (the H_base argument of aloco_sync).
+ *
+ * Rules followed (App. A.1-A.3; Tab. AutoLoCo configuration):
+ *   - the recipe horizon H_base runs through the inner-lr warm-up; from the
+ *     interval that completes warm-up, ref_bootstrap finite intervals set
+ *     D_ref, C_ref to geometric means; variability_intervals more intervals
+ *     fill the residual histories; then one monitoring interval;
+ *   - residuals r_D = log(sqrt(D)/(sqrt(D_ref) xi + eps) + eps),
+ *     r_C = -log(C/(C_ref + eps) + eps), xi = Lambda/(Lambda_ref + eps)
+ *     (Eqs. adaptive-h-lr-mass, adaptive-h-core-residuals); centre = median,
+ *     scale = MAD of at most 16 residuals; z = max of the positive parts
+ *     over the scales (Eq. adaptive-h-core-deviation);
+ *   - z < 1.5 supports an increase, < 2.5 is reference consistent, < 4.0 is
+ *     a moderate deviation (two in a row reduce by 1.20), otherwise severe
+ *     (reduce by 1.50); a non-finite statistic takes the severe path, and
+ *     consecutive severe or invalid intervals fall back to H_min
+ *     (Tab. adaptive-h-assessment); only the first reference estimate skips
+ *     non-finite intervals instead ("two finite intervals", App. A.1);
+ *   - a supported monitoring interval proposes the longest admissible horizon
+ *     whose previewed accumulated inner lr is at most 1.15 times that of the
+ *     accepted horizon, or, while a rejected-horizon bound is active, the
+ *     admissible horizon nearest the geometric midpoint of accepted and
+ *     bound; the bound retires once its previewed exposure falls to 0.90 of
+ *     the value stored when it was set;
+ *   - a candidate is adopted after one supported interval, or two intervals
+ *     of which the first is consistent and the second supported or
+ *     consistent; a moderate or severe candidate interval is rejected and the
+ *     accepted horizon restored; after adoption, return or reduction the
+ *     reference is re-estimated (one interval) and its variability measured
+ *     again before the next proposal;
+ *   - token mapper: M_base = median token mass of the first three recipe-
+ *     horizon intervals, n_hat = EMA (beta) of tokens per step; the step
+ *     horizon is the multiple of q_H nearest M_base H_tok / (H_base n_hat),
+ *     the identity before calibration (Eq. adaptive-h-token-mapping).
+ * Horizons are admissible when they are multiples of q_H within
+ * [H_min, H_max]; ties between two nearest horizons take the smaller.
+ * ---------------------------------------------------------------------- */
+
+#define ALOCO_CTRL_HISTORY 16
+
+typedef enum {
+    ALOCO_ASSESS_NONE = 0,        /* not assessed (warm-up, calibration)   */
+    ALOCO_ASSESS_SUPPORTED = 1,   /* z < thr_candidate                     */
+    ALOCO_ASSESS_CONSISTENT = 2,  /* z < thr_moderate                      */
+    ALOCO_ASSESS_MODERATE = 3,    /* z < thr_severe                        */
+    ALOCO_ASSESS_SEVERE = 4,      /* z >= thr_severe                       */
+    ALOCO_ASSESS_INVALID = 5      /* a required statistic is not finite    */
+} aloco_assessment;
+
+typedef enum {
+    ALOCO_PHASE_WARMUP = 0,
+    ALOCO_PHASE_REFERENCE = 1,    /* estimating D_ref, C_ref, Lambda_ref   */
+    ALOCO_PHASE_VARIABILITY = 2,  /* filling the residual histories        */
+    ALOCO_PHASE_MONITOR = 3,      /* at the accepted horizon               */
+    ALOCO_PHASE_CANDIDATE = 4,    /* first interval at a longer candidate  */
+    ALOCO_PHASE_CONFIRM = 5       /* second interval at the candidate      */
+} aloco_ctrl_phase;
+
+/* Controller settings.  aloco_ctrl_default_cfg() fills the paper's shared
+ * settings (Tab. AutoLoCo configuration) and the readings where the paper
+ * gives no value (ref_ema, mad_scale, scale_floor, severe_fallback). */
+typedef struct aloco_ctrl_cfg {
+    int64_t H_base;               /* recipe token horizon (500 C4, 100 SFT)*/
+    int64_t H_min, H_max;         /* token-horizon bounds                  */
+    int64_t q_H;                  /* horizon quantum                       */
+    int64_t warmup_steps;         /* inner-lr warm-up held at H_base       */
+    double beta_tok;              /* token-density EMA coefficient, 0.9    */
+    double thr_candidate;         /* 1.5 */
+    double thr_moderate;          /* 2.5 */
+    double thr_severe;            /* 4.0 */
+    double exposure_mult;         /* 1.15 */
+    double div_moderate;          /* 1.20 */
+    double div_severe;            /* 1.50 */
+    double retire_frac;           /* 0.90 */
+    double ref_ema;               /* weight of a new interval in the
+                                     log-space EMA of D_ref, C_ref (0.1)   */
+    double mad_scale;             /* scale = mad_scale * MAD (1.4826)      */
+    double scale_floor;           /* lower bound of a residual scale (1e-3)*/
+    double eps;                   /* 1e-8 */
+    int32_t mapper_bootstrap;     /* 3 */
+    int32_t ref_bootstrap;        /* 2 */
+    int32_t variability_intervals;/* 3 */
+    int32_t severe_fallback;      /* consecutive severe/invalid -> H_min (2)*/
+} aloco_ctrl_cfg_t;
+
+/* Controller state: plain data, so it can be checkpointed by copying the
+ * bytes (aloco_ctrl_save / aloco_ctrl_load add a version check). */
+typedef struct aloco_ctrl_state {
+    int32_t version;
+    int32_t phase;                /* aloco_ctrl_phase of the next interval */
+    int64_t intervals;            /* completed intervals observed          */
+    int64_t H_acc;                /* accepted token horizon                */
+    int64_t H_next;               /* token horizon of the next interval    */
+    int64_t H_cand;               /* candidate under evaluation, 0 if none */
+    int64_t bound;                /* rejected-horizon bound, 0 if none     */
+    double bound_lam;             /* Lambda observed when the bound was set*/
+    int32_t phase_count;          /* intervals completed in this phase     */
+    int32_t ref_needed;           /* intervals the reference estimate uses */
+    int32_t moderate_run;
+    int32_t severe_run;
+    double log_D_ref, log_C_ref, lam_ref;
+    double sum_log_D, sum_log_C;  /* reference bootstrap accumulators      */
+    int32_t n_hist, head;         /* residual ring (shared by D and C)     */
+    double hist_D[ALOCO_CTRL_HISTORY], hist_C[ALOCO_CTRL_HISTORY];
+    int32_t mapper_n, calibrated;
+    double mapper_mass[8];
+    double M_base, n_hat;
+    double last_z, last_r_D, last_r_C;
+    int32_t last_assessment;
+    int32_t referenced;           /* 1 once a reference profile was set    */
+} aloco_ctrl_state_t;
+
+/* One completed interval. */
+typedef struct aloco_interval_obs {
+    double D;                     /* local-drift energy (aloco_stats_t.D)  */
+    double C;                     /* aggregation coherence                 */
+    double lam;                   /* accumulated inner lr of the interval  */
+    double tokens;                /* non-padding tokens M_t it processed   */
+    int64_t H_step;               /* steps it executed                     */
+    int64_t step_end;             /* global inner step at which it ended   */
+} aloco_interval_obs_t;
+
+/* The controller's answer for the next interval. */
+typedef struct aloco_ctrl_decision {
+    int64_t H_tok;                /* token horizon H_{t+1}^tok             */
+    int64_t H_step;               /* executable steps H_{t+1}^step         */
+    int64_t H_ref_step;           /* steps of one base token interval      */
+    int32_t assessment;           /* of the completed interval             */
+    int32_t phase;                /* aloco_ctrl_phase of the next interval */
+    double z, r_D, r_C;           /* z_t^max and residuals (0 if none)     */
+} aloco_ctrl_decision_t;
+
+/* Fill *cfg with the paper's settings for a recipe horizon H_base, bounds
+ * [H_min, H_max], quantum q_H and an inner-lr warm-up of warmup_steps. */
+void aloco_ctrl_default_cfg(aloco_ctrl_cfg_t *cfg, int64_t H_base,
+                            int64_t H_min, int64_t H_max, int64_t q_H,
+                            int64_t warmup_steps);
+
+/* Start a run: the first interval executes H_base.  Returns ALOCO_ERR_ARG
+ * for an inconsistent cfg (H_min <= H_base <= H_max, all multiples of q_H,
+ * thresholds increasing, ...). */
+int aloco_ctrl_init(aloco_ctrl_state_t *state, const aloco_ctrl_cfg_t *cfg,
+                    aloco_ctrl_decision_t *first);
+
+/* Feed one completed interval and choose the next one (App. A).  The
+ * schedule is used to preview accumulated inner learning rates from
+ * obs->step_end.  state is updated in place. */
+int aloco_select_interval(aloco_ctrl_state_t *state,
+                          const aloco_ctrl_cfg_t *cfg,
+                          const aloco_interval_obs_t *obs,
+                          const aloco_schedule_t *schedule,
+                          aloco_ctrl_decision_t *out);
+
+/* Serialise / restore a controller state (checkpoint and resume).  save
+ * writes aloco_ctrl_state_bytes() bytes; load checks the version. */
+size_t aloco_ctrl_state_bytes(void);
+int aloco_ctrl_save(const aloco_ctrl_state_t *state, void *buf, size_t len);
+int aloco_ctrl_load(aloco_ctrl_state_t *state, const void *buf, size_t len);
+
 /* Block partials the scratch of aloco_sync_noalloc can hold. */
 #define ALOCO_NOALLOC_MAX_BLOCKS 2048
 

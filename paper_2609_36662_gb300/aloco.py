@@ -31,7 +31,15 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
 # Names declared in include/aloco.h (checked by the ABI test).
 EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
            "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc",
+           "aloco_ctrl_default_cfg", "aloco_ctrl_init", "aloco_select_interval",
+           "aloco_ctrl_state_bytes", "aloco_ctrl_save", "aloco_ctrl_load",
            "aloco_last_error", "aloco_shutdown", "aloco_version")
+
+CTRL_HISTORY = 16
+ASSESS_NONE, ASSESS_SUPPORTED, ASSESS_CONSISTENT, ASSESS_MODERATE, \
+    ASSESS_SEVERE, ASSESS_INVALID = range(6)
+PHASE_WARMUP, PHASE_REFERENCE, PHASE_VARIABILITY, PHASE_MONITOR, \
+    PHASE_CANDIDATE, PHASE_CONFIRM = range(6)
 
 
 class Schedule(ctypes.Structure):
@@ -81,6 +89,51 @@ class Stats(ctypes.Structure):
                 "pass_used": self.pass_used}
 
 
+_i64, _i32, _dbl = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
+
+
+class CtrlCfg(ctypes.Structure):
+    _fields_ = [("H_base", _i64), ("H_min", _i64), ("H_max", _i64),
+                ("q_H", _i64), ("warmup_steps", _i64), ("beta_tok", _dbl),
+                ("thr_candidate", _dbl), ("thr_moderate", _dbl),
+                ("thr_severe", _dbl), ("exposure_mult", _dbl),
+                ("div_moderate", _dbl), ("div_severe", _dbl),
+                ("retire_frac", _dbl), ("ref_ema", _dbl), ("mad_scale", _dbl),
+                ("scale_floor", _dbl), ("eps", _dbl),
+                ("mapper_bootstrap", _i32), ("ref_bootstrap", _i32),
+                ("variability_intervals", _i32), ("severe_fallback", _i32)]
+
+
+class CtrlState(ctypes.Structure):
+    _fields_ = [("version", _i32), ("phase", _i32), ("intervals", _i64),
+                ("H_acc", _i64), ("H_next", _i64), ("H_cand", _i64),
+                ("bound", _i64), ("bound_lam", _dbl), ("phase_count", _i32),
+                ("ref_needed", _i32), ("moderate_run", _i32),
+                ("severe_run", _i32), ("log_D_ref", _dbl),
+                ("log_C_ref", _dbl), ("lam_ref", _dbl), ("sum_log_D", _dbl),
+                ("sum_log_C", _dbl), ("n_hist", _i32), ("head", _i32),
+                ("hist_D", _dbl * CTRL_HISTORY),
+                ("hist_C", _dbl * CTRL_HISTORY), ("mapper_n", _i32),
+                ("calibrated", _i32), ("mapper_mass", _dbl * 8),
+                ("M_base", _dbl), ("n_hat", _dbl), ("last_z", _dbl),
+                ("last_r_D", _dbl), ("last_r_C", _dbl),
+                ("last_assessment", _i32), ("referenced", _i32)]
+
+
+class IntervalObs(ctypes.Structure):
+    _fields_ = [("D", _dbl), ("C", _dbl), ("lam", _dbl), ("tokens", _dbl),
+                ("H_step", _i64), ("step_end", _i64)]
+
+
+class CtrlDecision(ctypes.Structure):
+    _fields_ = [("H_tok", _i64), ("H_step", _i64), ("H_ref_step", _i64),
+                ("assessment", _i32), ("phase", _i32), ("z", _dbl),
+                ("r_D", _dbl), ("r_C", _dbl)]
+
+    def as_dict(self):
+        return {n: getattr(self, n) for n, _ in self._fields_}
+
+
 class AlocoError(RuntimeError):
     def __init__(self, status: int, message: str):
         super().__init__(f"aloco status {status}: {message}")
@@ -124,6 +177,23 @@ def load():
     lib.aloco_sync_noalloc.argtypes = sync_args + [ctypes.POINTER(Opts),
                                                    ctypes.POINTER(Stats)]
     lib.aloco_sync_noalloc.restype = i32
+    P = ctypes.POINTER
+    lib.aloco_ctrl_default_cfg.argtypes = [P(CtrlCfg), i64, i64, i64, i64,
+                                           i64]
+    lib.aloco_ctrl_default_cfg.restype = None
+    lib.aloco_ctrl_init.argtypes = [P(CtrlState), P(CtrlCfg),
+                                    P(CtrlDecision)]
+    lib.aloco_ctrl_init.restype = i32
+    lib.aloco_select_interval.argtypes = [P(CtrlState), P(CtrlCfg),
+                                          P(IntervalObs), P(Schedule),
+                                          P(CtrlDecision)]
+    lib.aloco_select_interval.restype = i32
+    lib.aloco_ctrl_state_bytes.argtypes = []
+    lib.aloco_ctrl_state_bytes.restype = ctypes.c_size_t
+    lib.aloco_ctrl_save.argtypes = [P(CtrlState), vp, ctypes.c_size_t]
+    lib.aloco_ctrl_save.restype = i32
+    lib.aloco_ctrl_load.argtypes = [P(CtrlState), vp, ctypes.c_size_t]
+    lib.aloco_ctrl_load.restype = i32
     lib.aloco_last_error.argtypes = []
     lib.aloco_last_error.restype = ctypes.c_char_p
     lib.aloco_shutdown.argtypes = []
@@ -230,3 +300,51 @@ def sync(global_, momentum, locals_, *, H_sel: int, H_base: int, step: int,
 def shutdown():
     if _lib is not None:
         _lib.aloco_shutdown()
+
+
+class Controller:
+    """The host interval controller (aloco_select_interval) with its state
+    and settings."""
+
+    def __init__(self, H_base: int, H_min: int, H_max: int, q_H: int,
+                 warmup_steps: int, schedule: Schedule, **overrides):
+        lib = load()
+        self.cfg = CtrlCfg()
+        lib.aloco_ctrl_default_cfg(ctypes.byref(self.cfg), H_base, H_min,
+                                   H_max, q_H, warmup_steps)
+        for k, val in overrides.items():
+            setattr(self.cfg, k, val)
+        self.schedule = schedule
+        self.state = CtrlState()
+        d = CtrlDecision()
+        rc = lib.aloco_ctrl_init(ctypes.byref(self.state),
+                                 ctypes.byref(self.cfg), ctypes.byref(d))
+        if rc != OK:
+            raise AlocoError(rc, last_error())
+        self.decision = d
+
+    def observe(self, D: float, C: float, lam: float, tokens: float,
+                H_step: int, step_end: int) -> CtrlDecision:
+        obs = IntervalObs(D, C, lam, tokens, H_step, step_end)
+        d = CtrlDecision()
+        rc = load().aloco_select_interval(
+            ctypes.byref(self.state), ctypes.byref(self.cfg),
+            ctypes.byref(obs), ctypes.byref(self.schedule), ctypes.byref(d))
+        if rc != OK:
+            raise AlocoError(rc, last_error())
+        self.decision = d
+        return d
+
+    def save(self) -> bytes:
+        n = load().aloco_ctrl_state_bytes()
+        buf = ctypes.create_string_buffer(n)
+        rc = load().aloco_ctrl_save(ctypes.byref(self.state), buf, n)
+        if rc != OK:
+            raise AlocoError(rc, last_error())
+        return buf.raw
+
+    def load_state(self, blob: bytes):
+        buf = ctypes.create_string_buffer(blob, len(blob))
+        rc = load().aloco_ctrl_load(ctypes.byref(self.state), buf, len(blob))
+        if rc != OK:
+            raise AlocoError(rc, last_error())

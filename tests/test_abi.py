@@ -56,6 +56,10 @@ def test_struct_layout_matches_c(tmp_path):
 int main(void) {
   printf("%zu %zu %zu %zu\n", sizeof(aloco_schedule_t), sizeof(aloco_opts_t),
          sizeof(aloco_correction_t), sizeof(aloco_stats_t));
+  printf("%zu %zu %zu %zu %zu %zu\n", sizeof(aloco_ctrl_cfg_t),
+         sizeof(aloco_ctrl_state_t), sizeof(aloco_interval_obs_t),
+         sizeof(aloco_ctrl_decision_t), offsetof(aloco_ctrl_state_t, hist_C),
+         offsetof(aloco_ctrl_state_t, referenced));
   printf("%zu %zu %zu %zu %zu %zu %zu\n", offsetof(aloco_opts_t, pass), offsetof(aloco_opts_t, stream),
          offsetof(aloco_stats_t, corr), offsetof(aloco_stats_t, nonfinite),
          offsetof(aloco_stats_t, kernel_ms), offsetof(aloco_schedule_t, peak_lr),
@@ -69,7 +73,11 @@ int main(void) {
     lines = subprocess.run([str(exe)], capture_output=True, text=True,
                            check=True).stdout.split("\n")
     sizes = list(map(int, lines[0].split()))
-    offs = list(map(int, lines[1].split()))
+    ctrl = list(map(int, lines[1].split()))
+    offs = list(map(int, lines[2].split()))
+    assert ctrl == [ctypes.sizeof(A.CtrlCfg), ctypes.sizeof(A.CtrlState),
+                    ctypes.sizeof(A.IntervalObs), ctypes.sizeof(A.CtrlDecision),
+                    A.CtrlState.hist_C.offset, A.CtrlState.referenced.offset]
     assert sizes == [ctypes.sizeof(A.Schedule), ctypes.sizeof(A.Opts),
                      ctypes.sizeof(A.Correction), ctypes.sizeof(A.Stats)]
     assert offs == [A.Opts.pass_.offset, A.Opts.stream.offset,
