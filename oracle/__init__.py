@@ -74,6 +74,13 @@ def _load():
                               vp, vp, vp]
     lib.orc_stats.restype = None
     lib.orc_stats.argtypes = [dp, dbl, i32, dbl, dp]
+    lib.orc_int8_blocks.restype = i64
+    lib.orc_int8_blocks.argtypes = [vp, i32]
+    lib.orc_int8_encode.restype = None
+    lib.orc_int8_encode.argtypes = [vp, vp, i32, vp, vp, vp]
+    lib.orc_int8_round.restype = i64
+    lib.orc_int8_round.argtypes = [vp, vp, vp, i32, vp, i32, i32, dbl, dbl,
+                                   dbl, vp, vp, vp, dp, dp]
     _lib = lib
     return lib
 
@@ -208,3 +215,64 @@ def sync_round(g, v, xs, dtype, schedule: Schedule, step: int, H_sel: int,
                                     corr.inv_norm)
     st.update(g=g_out, v=v_out, x=x_out, nonfinite=nf, corr=corr)
     return st
+
+
+# ------------------------------------------------ INT8 communication (App. G.1)
+
+INT8_BLOCK = 4096
+
+
+def _parts(parts, N):
+    p = np.ascontiguousarray([N] if parts is None else parts, dtype=np.int64)
+    assert int(p.sum()) == N, "parts must add up to the vector length"
+    return p
+
+
+def int8_blocks(parts) -> int:
+    p = np.ascontiguousarray(parts, dtype=np.int64)
+    return int(_load().orc_int8_blocks(_ptr(p), len(p)))
+
+
+def int8_payload_bytes(parts) -> int:
+    """Logical bytes one worker sends per sync: one int8 per element and one
+    fp32 scale per block."""
+    return int(np.sum(parts)) + 4 * int8_blocks(parts)
+
+
+def int8_encode(y, parts=None):
+    """Blockwise INT8 codec of an fp32 vector: (codes int8, scales float32
+    per block, decoded float32)."""
+    y = np.ascontiguousarray(y, dtype=np.float32)
+    p = _parts(parts, y.shape[0])
+    nb = int8_blocks(p)
+    codes = np.empty(y.shape[0], np.int8)
+    scales = np.empty(nb, np.float32)
+    dec = np.empty(y.shape[0], np.float32)
+    _load().orc_int8_encode(_ptr(y), _ptr(p), len(p), _ptr(codes),
+                            _ptr(scales), _ptr(dec))
+    return codes, scales, dec
+
+
+def int8_round(g, v, xs, dtype, parts, mu_t, eta_out, inv_norm, eps=1e-8):
+    """The outer round with INT8-communicated pseudo-gradients: D from the
+    pre-quantisation pseudo-gradients, C from the decoded aggregate."""
+    g, v, xs, N = _check_inputs(g, v, xs, dtype)
+    p = _parts(parts, N)
+    M = len(xs)
+    g_out = np.empty(N, np.float64)
+    v_out = np.empty(N, np.float64)
+    rdt = np.float32 if dtype == F32 else np.uint16
+    x_out = [np.empty(N, rdt) for _ in range(M)]
+    E = (ctypes.c_double * M)()
+    B = ctypes.c_double(0.0)
+    ptrs = (ctypes.c_void_p * M)(*[_ptr(x) for x in xs])
+    optrs = (ctypes.c_void_p * M)(*[_ptr(x) for x in x_out])
+    nf = _load().orc_int8_round(_ptr(g), _ptr(v), ptrs, dtype, _ptr(p),
+                                len(p), M, mu_t, eta_out, inv_norm,
+                                _ptr(g_out), _ptr(v_out), optrs, E,
+                                ctypes.byref(B))
+    out = (ctypes.c_double * 2)()
+    _load().orc_stats(E, B.value, M, eps, out)
+    return {"D": out[0], "C": out[1], "mean_sq_norm": B.value,
+            "drift": list(E), "g": g_out, "v": v_out, "x": x_out,
+            "nonfinite": int(nf)}

@@ -267,3 +267,144 @@ void orc_stats(const double *E, double B, int M, double eps, double *out)
     out[0] = D;
     out[1] = (double)M * B / (D + eps);
 }
+
+/* ---- INT8 pseudo-gradient communication (App. G.1) ----
+ *
+ * Blocks: each tensor part (a contiguous range of the flattened vector,
+ * parts given by their sizes) is cut into consecutive blocks of at most 4096
+ * elements starting at the part's first element.
+ *
+ * Codec, in FP32 as the appendix states: scale = max|y| / 127 (1 for an
+ * all-zero block; kept within [FLT_MIN, FLT_MAX / 127] so that it neither
+ * underflows to zero nor overflows on reconstruction); q = y / scale rounded
+ * to the nearest integer, ties to even, clipped to [-127, 127] (a NaN
+ * quotient gives q = 0 and the NaN stays in the scale); decode = q * scale.
+ * Aggregation: decoded worker contributions are added in FP32 in worker
+ * order and divided by M; the mean is encoded and decoded once.
+ */
+#include <float.h>
+
+#define ORC_INT8_BLOCK 4096
+
+int64_t orc_int8_blocks(const int64_t *parts, int n_parts)
+{
+    int64_t nb = 0;
+    for (int p = 0; p < n_parts; ++p)
+        nb += (parts[p] + ORC_INT8_BLOCK - 1) / ORC_INT8_BLOCK;
+    return nb;
+}
+
+static float orc_int8_scale(const float *y, int64_t n)
+{
+    float amax = 0.0f;
+    for (int64_t i = 0; i < n; ++i) {
+        float a = fabsf(y[i]);
+        if (isnan(a)) return a;           /* NaN propagates through the scale */
+        if (a > amax) amax = a;
+    }
+    if (amax == 0.0f) return 1.0f;
+    float s = amax / 127.0f;
+    if (s < FLT_MIN) s = FLT_MIN;
+    if (s > FLT_MAX / 127.0f) s = FLT_MAX / 127.0f;
+    return s;
+}
+
+static int8_t orc_int8_code(float y, float s)
+{
+    float t = rintf(y / s);
+    if (isnan(t)) return 0;
+    if (t > 127.0f) t = 127.0f;
+    if (t < -127.0f) t = -127.0f;
+    return (int8_t)t;
+}
+
+/* Encode a vector blockwise: codes[N], scales[n_blocks], decoded[N]. */
+void orc_int8_encode(const float *y, const int64_t *parts, int n_parts,
+                     int8_t *codes, float *scales, float *decoded)
+{
+    int64_t off = 0, b = 0;
+    for (int p = 0; p < n_parts; ++p) {
+        for (int64_t s0 = 0; s0 < parts[p]; s0 += ORC_INT8_BLOCK, ++b) {
+            int64_t n = parts[p] - s0 < ORC_INT8_BLOCK ? parts[p] - s0
+                                                       : ORC_INT8_BLOCK;
+            const float *yb = y + off + s0;
+            float s = orc_int8_scale(yb, n);
+            scales[b] = s;
+            for (int64_t i = 0; i < n; ++i) {
+                int8_t q = orc_int8_code(yb[i], s);
+                codes[off + s0 + i] = q;
+                decoded[off + s0 + i] = (float)q * s;
+            }
+        }
+        off += parts[p];
+    }
+}
+
+/* One outer round with INT8-communicated pseudo-gradients over the whole
+ * vector (length = sum of parts).  Per block:
+ *   Delta_m = fl32(g - x_m)               (the FP32 pseudo-gradient sent)
+ *   E[m]   += (g - x_m)^2 in double       (D from the pre-quantisation Delta)
+ *   mean    = fl32(sum_m decode(encode(Delta_m))) / M       (FP32, in order)
+ *   Dq      = decode(encode(mean))        (the aggregate every worker gets)
+ *   B      += Dq^2 in double              (C from the decoded aggregate)
+ *   v' = mu v + Dq inv ; d = Dq inv + mu v' ; g' = g - eta d   (double)
+ * Outputs as orc_pass2 (g_out, v_out double; x_out in storage type, may be
+ * NULL).  E, B accumulate.  Returns the number of non-finite elements. */
+int64_t orc_int8_round(const float *g, const float *v, const void *const *x,
+                       int dtype, const int64_t *parts, int n_parts, int M,
+                       double mu_t, double eta_out, double inv_norm,
+                       double *g_out, double *v_out, void *const *x_out,
+                       double *E, double *B)
+{
+    float delta[ORC_INT8_BLOCK], dec[ORC_INT8_BLOCK], sum[ORC_INT8_BLOCK];
+    int8_t q[ORC_INT8_BLOCK];
+    int64_t nonfinite = 0, off = 0;
+    for (int p = 0; p < n_parts; ++p) {
+        for (int64_t s0 = 0; s0 < parts[p]; s0 += ORC_INT8_BLOCK) {
+            int64_t n = parts[p] - s0 < ORC_INT8_BLOCK ? parts[p] - s0
+                                                       : ORC_INT8_BLOCK;
+            int64_t base = off + s0;
+            for (int64_t i = 0; i < n; ++i) sum[i] = 0.0f;
+            for (int m = 0; m < M; ++m) {
+                for (int64_t i = 0; i < n; ++i) {
+                    double xd = orc_replica(x[m], dtype, base + i);
+                    double dd = (double)g[base + i] - xd;
+                    E[m] += dd * dd;
+                    delta[i] = g[base + i] - (float)xd;
+                }
+                float s = orc_int8_scale(delta, n);
+                for (int64_t i = 0; i < n; ++i) {
+                    float d = (float)orc_int8_code(delta[i], s) * s;
+                    sum[i] = m == 0 ? d : sum[i] + d;
+                }
+            }
+            for (int64_t i = 0; i < n; ++i) sum[i] = sum[i] / (float)M;
+            float s = orc_int8_scale(sum, n);
+            for (int64_t i = 0; i < n; ++i) {
+                q[i] = orc_int8_code(sum[i], s);
+                dec[i] = (float)q[i] * s;
+            }
+            for (int64_t i = 0; i < n; ++i) {
+                int64_t e = base + i;
+                double dq = (double)dec[i];
+                *B += dq * dq;
+                double dtil = dq * inv_norm;
+                double vn = mu_t * (double)v[e] + dtil;
+                double dn = dtil + mu_t * vn;
+                double gp = (double)g[e] - eta_out * dn;
+                g_out[e] = gp;
+                v_out[e] = vn;
+                if (!isfinite(gp) || !isfinite(vn)) ++nonfinite;
+                for (int m = 0; m < M; ++m) {
+                    if (x_out == 0 || x_out[m] == 0) continue;
+                    if (dtype == 0)
+                        ((float *)x_out[m])[e] = (float)gp;
+                    else
+                        ((uint16_t *)x_out[m])[e] = orc_double_to_bf16(gp);
+                }
+            }
+        }
+        off += parts[p];
+    }
+    return nonfinite;
+}

@@ -65,6 +65,9 @@ LLAMA_1B = LlamaShape(layers=22, d_model=2048, heads=32, kv_heads=4,
                       ffn=5632, vocab=32000, tied=False)
 LLAMA_3B = LlamaShape(layers=26, d_model=3072, heads=24, kv_heads=8,
                       ffn=8192, vocab=32000, tied=False)
+# Llama-3.1-8B (the paper's fine-tuning model) for payload accounting.
+LLAMA31_8B = LlamaShape(layers=32, d_model=4096, heads=32, kv_heads=8,
+                        ffn=14336, vocab=128256, tied=False)
 
 
 @dataclass(frozen=True)
@@ -278,6 +281,12 @@ def _sigma_slice(segs, s, e, device):
         return float(parts[0][1])
     return torch.cat([torch.full((k,), sig, dtype=torch.float32,
                                  device=device) for k, sig in parts])
+
+
+def tensor_sizes(w: Workload) -> List[int]:
+    """Sizes of the tensor parts of the layout (one part for a flat
+    vector)."""
+    return [n for _, n, _, _ in _segments(w)]
 
 
 def tensor_boundaries(w: Workload) -> List[int]:
