@@ -316,7 +316,7 @@ def run_cuda(args, w):
                             s.total_steps)
     stream = torch.cuda.Stream(device)
 
-    # CPU baseline: the oracle on a bounded sample of round 0 (rank 0, N=1)
+    # CPU baseline: the oracle on a bounded sample of the first outer round (rank 0, N=1)
     cpu_baseline = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         step0, h0 = rounds[0]
@@ -329,6 +329,7 @@ def run_cuda(args, w):
                                   f"({t:.1f} s), scaled to a full round"}
 
     opts = A.default_opts(time_kernel=1, pass_=PASSES[args.pass_])
+    parts = W.tensor_sizes(w)
     step_ms, kern_ms, statuses = [], [], []
     ev = [(torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in rounds]
@@ -339,9 +340,15 @@ def run_cuda(args, w):
             with torch.cuda.stream(stream):
                 W.fill_replicas(w, g, xs, k)      # untimed: the inner loops
         ev[k][0].record(stream)
-        st = A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step,
-                    schedule=sched, outer_lr=w.outer_lr,
-                    outer_beta=w.outer_beta, opts=opts, stream=stream)
+        if args.comm == "int8":
+            st = A.sync_int8(g, v, xs, parts=parts, H_sel=hsel,
+                             H_base=w.H_base, step=step, schedule=sched,
+                             outer_lr=w.outer_lr, outer_beta=w.outer_beta,
+                             opts=opts, stream=stream)
+        else:
+            st = A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step,
+                        schedule=sched, outer_lr=w.outer_lr,
+                        outer_beta=w.outer_beta, opts=opts, stream=stream)
         ev[k][1].record(stream)
         return st
 
@@ -367,7 +374,8 @@ def run_cuda(args, w):
     for k in range(args.warmup, args.warmup + args.steps):
         step_ms.append(ev[k][0].elapsed_time(ev[k][1]))
 
-    kernel_name = ("sync_tma_kernel" if st_first.get("pass_used") == 2
+    kernel_name = ("int8_round_kernel" if args.comm == "int8" else
+                   "sync_tma_kernel" if st_first.get("pass_used") == 2
                    else "sync_kernel")
     ms_step = statistics.mean(step_ms)
     ms_step = reduce_max(ms_step, world, device)
@@ -379,7 +387,7 @@ def run_cuda(args, w):
     # end to end through the C ABI with host buffers: H2D of the round's
     # inputs from pinned memory, the round, D2H of theta' and v'
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and args.comm == "fp32":
         e2e = run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device)
 
     if rank == 0:
@@ -390,7 +398,7 @@ def run_cuda(args, w):
             "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded; Llama-shaped parameter set, "
                     "shared/private drift noise)",
-            "config": config_block(w),
+            "config": dict(config_block(w), comm=args.comm),
             "rounds_per_s_per_gpu": 1e3 / ms_step,
             "elem_per_s": value * w.numel * w.M,
             "kernel_ms": ms_kern,
@@ -486,6 +494,9 @@ def main(argv=None):
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--pass", dest="pass_", choices=sorted(PASSES),
                    default="auto", help="which fused kernel runs the round")
+    p.add_argument("--comm", choices=["fp32", "int8"], default="fp32",
+                   help="int8: the round with INT8-communicated "
+                        "pseudo-gradients (App. G.1)")
     p.add_argument("--list", action="store_true")
     args = p.parse_args(argv)
     table = workloads_by_name()

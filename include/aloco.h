@@ -234,6 +234,51 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
                   aloco_stats_t *stats_out);
 
 /* ------------------------------------------------------------------------
+ * INT8 pseudo-gradient communication (App. G.1).
+ *
+ * Blocks: the flattened vector is a sequence of tensor parts (part_sizes,
+ * n_parts <= 1024; NULL means one part of N); each part is cut into
+ * consecutive blocks of at most 4096 elements starting at its first
+ * element.  Codec, in FP32: scale = max|y| / 127 per block (1 for an all-zero
+ * block; kept within [FLT_MIN, FLT_MAX / 127]), q = y / scale rounded to the
+ * nearest integer with ties to even and clipped to [-127, 127], decoded value
+ * q * scale.  One worker's payload per sync is N bytes of codes plus 4 bytes
+ * per block (aloco_int8_num_blocks).
+ * ---------------------------------------------------------------------- */
+
+/* Number of codec blocks of a vector made of the given parts, or -1. */
+int64_t aloco_int8_num_blocks(const int64_t *part_sizes, int n_parts);
+
+/* Encode an fp32 device vector x[N]: codes[N] (int8), scales[num_blocks]
+ * (fp32) and, when decoded != NULL, decoded[N] = codes * scale.  Device
+ * buffers; enqueued on `stream` (cudaStream_t, NULL = default) without
+ * waiting. */
+int aloco_int8_encode(const float *x, size_t N, const int64_t *part_sizes,
+                      int n_parts, int8_t *codes, float *scales,
+                      float *decoded, void *stream);
+
+/* Decode codes[N] with scales[num_blocks] into out[N] (device buffers,
+ * enqueued on `stream`). */
+int aloco_int8_decode(const int8_t *codes, const float *scales, size_t N,
+                      const int64_t *part_sizes, int n_parts, float *out,
+                      void *stream);
+
+/* One outer round with INT8-communicated pseudo-gradients (App. G.1): every
+ * worker's FP32 pseudo-gradient is encoded and decoded blockwise, the decoded
+ * contributions are averaged in FP32 (in worker order), the mean is encoded
+ * and decoded once, and that aggregate drives the corrected Nesterov step and
+ * the replica reset.  D_t and the drift energies use the pre-quantisation
+ * pseudo-gradients, C_t and ||Dbar||^2 the decoded aggregate.  Arguments as
+ * aloco_sync_ex plus the parts; M <= 16; opts->pass and blocks_per_sm do not
+ * apply (one kernel runs it). */
+int aloco_sync_int8(float *global, float *momentum, void *const *locals,
+                    size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                    int64_t H_base, int64_t step,
+                    const aloco_schedule_t *schedule, double outer_lr,
+                    double outer_beta, const int64_t *part_sizes, int n_parts,
+                    const aloco_opts_t *opts, aloco_stats_t *stats_out);
+
+/* ------------------------------------------------------------------------
  * Interval controller (Sec. 3.1; App. A).  Host-only and scalar: after each
  * completed interval it takes that interval's D_t, C_t, accumulated inner
  * learning rate and token count, assesses them against the accepted-horizon

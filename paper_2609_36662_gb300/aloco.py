@@ -31,6 +31,8 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
 # Names declared in include/aloco.h (checked by the ABI test).
 EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
            "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc",
+           "aloco_sync_int8", "aloco_int8_num_blocks", "aloco_int8_encode",
+           "aloco_int8_decode",
            "aloco_ctrl_default_cfg", "aloco_ctrl_init", "aloco_select_interval",
            "aloco_ctrl_state_bytes", "aloco_ctrl_save", "aloco_ctrl_load",
            "aloco_last_error", "aloco_shutdown", "aloco_version")
@@ -178,6 +180,15 @@ def load():
                                                    ctypes.POINTER(Stats)]
     lib.aloco_sync_noalloc.restype = i32
     P = ctypes.POINTER
+    lib.aloco_sync_int8.argtypes = sync_args + [vp, i32, P(Opts), P(Stats)]
+    lib.aloco_sync_int8.restype = i32
+    lib.aloco_int8_num_blocks.argtypes = [vp, i32]
+    lib.aloco_int8_num_blocks.restype = i64
+    lib.aloco_int8_encode.argtypes = [vp, ctypes.c_size_t, vp, i32, vp, vp, vp,
+                                      vp]
+    lib.aloco_int8_encode.restype = i32
+    lib.aloco_int8_decode.argtypes = [vp, vp, ctypes.c_size_t, vp, i32, vp, vp]
+    lib.aloco_int8_decode.restype = i32
     lib.aloco_ctrl_default_cfg.argtypes = [P(CtrlCfg), i64, i64, i64, i64,
                                            i64]
     lib.aloco_ctrl_default_cfg.restype = None
@@ -348,3 +359,94 @@ class Controller:
         rc = load().aloco_ctrl_load(ctypes.byref(self.state), buf, len(blob))
         if rc != OK:
             raise AlocoError(rc, last_error())
+
+
+# ------------------------------------------------ INT8 communication (App. G.1)
+
+def _parts_array(parts):
+    if parts is None:
+        return None, 0
+    arr = (ctypes.c_int64 * len(parts))(*[int(p) for p in parts])
+    return arr, len(parts)
+
+
+def int8_num_blocks(parts) -> int:
+    arr, n = _parts_array(parts)
+    nb = load().aloco_int8_num_blocks(arr, n)
+    if nb < 0:
+        raise AlocoError(ERR_ARG, last_error())
+    return nb
+
+
+def int8_payload_bytes(parts) -> int:
+    """Bytes one worker sends per sync: the codes plus one fp32 scale per
+    block."""
+    return int(sum(parts)) + 4 * int8_num_blocks(parts)
+
+
+def int8_encode(x, parts=None, want_decoded=True, stream=None):
+    """Blockwise INT8 codec of a contiguous float32 CUDA tensor; returns
+    (codes int8, scales float32, decoded float32 or None)."""
+    import torch
+    if x.dtype != torch.float32 or not x.is_cuda or not x.is_contiguous():
+        raise TypeError("x must be a contiguous float32 CUDA tensor")
+    N = x.numel()
+    nb = int8_num_blocks(parts if parts is not None else [N])
+    codes = torch.empty(N, dtype=torch.int8, device=x.device)
+    scales = torch.empty(nb, dtype=torch.float32, device=x.device)
+    dec = torch.empty_like(x) if want_decoded else None
+    s = stream if stream is not None else torch.cuda.current_stream(x.device)
+    arr, n = _parts_array(parts)
+    with torch.cuda.device(x.device):
+        rc = load().aloco_int8_encode(x.data_ptr(), N, arr, n,
+                                      codes.data_ptr(), scales.data_ptr(),
+                                      dec.data_ptr() if dec is not None
+                                      else None, s.cuda_stream)
+    if rc != OK:
+        raise AlocoError(rc, last_error())
+    return codes, scales, dec
+
+
+def int8_decode(codes, scales, parts=None, stream=None):
+    import torch
+    N = codes.numel()
+    out = torch.empty(N, dtype=torch.float32, device=codes.device)
+    s = stream if stream is not None else torch.cuda.current_stream(
+        codes.device)
+    arr, n = _parts_array(parts)
+    with torch.cuda.device(codes.device):
+        rc = load().aloco_int8_decode(codes.data_ptr(), scales.data_ptr(), N,
+                                      arr, n, out.data_ptr(), s.cuda_stream)
+    if rc != OK:
+        raise AlocoError(rc, last_error())
+    return out
+
+
+def sync_int8(global_, momentum, locals_, *, parts=None, H_sel: int,
+              H_base: int, step: int, schedule: Schedule, outer_lr: float,
+              outer_beta: float, opts: Optional[Opts] = None, stream=None,
+              raise_on_error=True):
+    """One outer round with INT8-communicated pseudo-gradients (in place on
+    torch CUDA tensors, like sync())."""
+    import torch
+    N = global_.numel()
+    rdt = locals_[0].dtype
+    dtype = F32 if rdt == torch.float32 else BF16
+    if opts is None:
+        opts = default_opts()
+    s = stream if stream is not None else torch.cuda.current_stream(
+        global_.device)
+    opts.stream = s.cuda_stream
+    M = len(locals_)
+    ptrs = (ctypes.c_void_p * M)(*[x.data_ptr() for x in locals_])
+    arr, n = _parts_array(parts)
+    st = Stats()
+    with torch.cuda.device(global_.device):
+        rc = load().aloco_sync_int8(global_.data_ptr(), momentum.data_ptr(),
+                                    ptrs, N, M, dtype, H_sel, H_base, step,
+                                    ctypes.byref(schedule), outer_lr,
+                                    outer_beta, arr, n, ctypes.byref(opts),
+                                    ctypes.byref(st))
+    if raise_on_error and rc not in (OK, ERR_NONFINITE):
+        raise AlocoError(rc, last_error())
+    return st.as_dict() | {"status": rc}

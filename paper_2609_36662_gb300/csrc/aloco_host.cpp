@@ -174,6 +174,8 @@ struct Workspace {
     unsigned long long *nf_total = nullptr;
     unsigned int *error = nullptr;
     unsigned int *ticket = nullptr;
+    char *i8 = nullptr;                   // INT8 round scratch (grown on demand)
+    size_t i8_cap = 0;
     double *host = nullptr;               // pinned readback of totals + nf
     cudaEvent_t ev0 = nullptr, ev1 = nullptr;
 };
@@ -324,15 +326,14 @@ void split_coef(double x, float *hi, float *lo) {
 }
 
 void finalize_stats(const double *totals, unsigned long long nf, int M,
-                    double eps, aloco_stats_t *st) {
+                    double eps, double b_scale, aloco_stats_t *st) {
     double sum = 0.0;
     for (int m = 0; m < M; ++m) {
         st->drift[m] = totals[m];
         sum += totals[m];
     }
     st->D = sum / (double)M;
-    // The pass accumulates S^2 with S = sum_m Delta_m = M * Dbar.
-    st->mean_sq_norm = totals[M] / ((double)M * (double)M);
+    st->mean_sq_norm = totals[M] * b_scale;
     st->C = (double)M * st->mean_sq_norm / (st->D + eps);
     st->nonfinite = (int64_t)nf;
 }
@@ -383,20 +384,49 @@ int aloco_sync(float *global, float *momentum, void *const *locals, size_t N,
                          stats_out);
 }
 
-int aloco_sync_ex(float *global, float *momentum, void *const *locals,
-                  size_t N, int M, aloco_dtype dtype, int64_t H_sel,
-                  int64_t H_base, int64_t step,
-                  const aloco_schedule_t *schedule, double outer_lr,
-                  double outer_beta, const aloco_opts_t *opts,
-                  aloco_stats_t *stats_out) {
+}  // extern "C"
+
+namespace {
+
+// Build the part table of an INT8 round (NULL parts: one part of N).
+int build_parts(const int64_t *parts, int n_parts, size_t N, aloco::Int8Parts *P) {
+    if (!parts) {
+        n_parts = 1;
+    } else if (n_parts < 1 || n_parts > aloco::kInt8MaxParts) {
+        return fail(ALOCO_ERR_ARG, "n_parts = %d outside [1, %d]", n_parts,
+                    aloco::kInt8MaxParts);
+    }
+    P->n_parts = n_parts;
+    P->off[0] = 0;
+    P->blk[0] = 0;
+    for (int p = 0; p < n_parts; ++p) {
+        const int64_t sz = parts ? parts[p] : (int64_t)N;
+        if (sz < 1) return fail(ALOCO_ERR_ARG, "part %d has size %lld", p, (long long)sz);
+        P->off[p + 1] = P->off[p] + sz;
+        P->blk[p + 1] = P->blk[p] + (sz + 4095) / 4096;
+    }
+    if ((size_t)P->off[n_parts] != N)
+        return fail(ALOCO_ERR_ARG, "parts add up to %lld, not N = %zu",
+                    (long long)P->off[n_parts], N);
+    return ALOCO_OK;
+}
+
+// One round: the plain pass (parts == NULL && !int8) or the INT8-
+// communicated pass.
+int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
+              int M, aloco_dtype dtype, int64_t H_sel, int64_t H_base,
+              int64_t step, const aloco_schedule_t *schedule, double outer_lr,
+              double outer_beta, bool int8, const int64_t *parts, int n_parts,
+              const aloco_opts_t *opts, aloco_stats_t *stats_out) {
     aloco_opts_t o;
     if (opts) o = *opts; else fill_default_opts(&o);
     aloco_stats_t local_stats;
     aloco_stats_t *st = stats_out ? stats_out : &local_stats;
 
     // ---------------------------------------------------- arguments
-    if (M < 1 || M > ALOCO_MAX_WORKERS)
-        return fail(ALOCO_ERR_ARG, "M = %d outside [1, %d]", M, ALOCO_MAX_WORKERS);
+    if (M < 1 || M > (int8 ? 16 : ALOCO_MAX_WORKERS))
+        return fail(ALOCO_ERR_ARG, "M = %d outside [1, %d]", M,
+                    int8 ? 16 : ALOCO_MAX_WORKERS);
     if (dtype != ALOCO_F32 && dtype != ALOCO_BF16)
         return fail(ALOCO_ERR_ARG, "unknown replica dtype %d", (int)dtype);
     if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
@@ -408,6 +438,9 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
     int rc = correction_impl(schedule, step, H_sel, H_base, outer_lr,
                              outer_beta, o, &corr);
     if (rc != ALOCO_OK) return rc;
+
+    static thread_local aloco::Int8Parts P;
+    if (int8 && (rc = build_parts(parts, n_parts, N, &P)) != ALOCO_OK) return rc;
 
     std::memset(st, 0, sizeof *st);
     st->corr = corr;
@@ -467,7 +500,8 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
     const int pack = aloco::pack_elems(dtype);
     a.n = (int64_t)N;
     a.nvec = (align_or & 15) == 0 ? (int64_t)(N / pack) : 0;
-    split_coef(corr.inv_norm / (double)M, &a.c_hi, &a.c_lo);
+    // plain pass: Dtil = (inv/M) sum_m Delta_m; INT8 pass: Dtil = inv * mean
+    split_coef(int8 ? corr.inv_norm : corr.inv_norm / (double)M, &a.c_hi, &a.c_lo);
     split_coef(corr.mu_t, &a.mu_hi, &a.mu_lo);
     split_coef(-corr.eta_out, &a.neg_eta_hi, &a.neg_eta_lo);
     a.M = M;
@@ -479,8 +513,28 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
 
     const int64_t work = a.nvec > 0 ? a.nvec : a.n;
     aloco::LaunchPlan plan;
-    const bool tma = aloco::use_tma(o.pass, M, dtype, a.nvec);
-    if (tma)
+    const bool tma = !int8 && aloco::use_tma(o.pass, M, dtype, a.nvec);
+    if (int8) {
+        // scratch of the two INT8 passes: per-block worker scales and the
+        // per-CTA drift energies of pass 1 (grown on demand, kept cached)
+        const size_t need = (size_t)P.blk[P.n_parts] * M * sizeof(float) + 256 +
+                            (size_t)ws->max_grid * 16 * sizeof(double);
+        if (ws->i8_cap < need) {
+            if (ws->i8) cudaFree(ws->i8);
+            ws->i8 = nullptr;
+            ws->i8_cap = 0;
+            e = cudaMalloc((void **)&ws->i8, need);
+            if (e != cudaSuccess) {
+                cudaGetLastError();
+                return fail(ALOCO_ERR_NOMEM, "INT8 scratch cudaMalloc(%zu): %s", need,
+                            cudaGetErrorString(e));
+            }
+            ws->i8_cap = need;
+        }
+        plan.grid = 0;
+        plan.block = 0;
+        plan.kernel = nullptr;
+    } else if (tma)
         e = dtype == ALOCO_F32 ? aloco::plan_sync_tma_f32(M, a.nvec, ws->sm_count, &plan)
                                : aloco::plan_sync_tma_bf16(M, a.nvec, ws->sm_count, &plan);
     else
@@ -498,9 +552,17 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
     cudaStream_t stream = (cudaStream_t)o.stream;
     if (o.time_kernel && (e = cudaEventRecord(ws->ev0, stream)) != cudaSuccess)
         return cuda_fail(e, "cudaEventRecord");
-    void *params[] = {&a};
-    e = cudaLaunchKernel(plan.kernel, dim3(plan.grid), dim3(plan.block), params,
-                         plan.smem, stream);
+    if (int8) {
+        double *e_rows = reinterpret_cast<double *>(ws->i8);
+        unsigned *bmax = reinterpret_cast<unsigned *>(
+            ws->i8 + (size_t)ws->max_grid * 16 * sizeof(double));
+        e = aloco::launch_int8_round(a, P, dtype, ws->sm_count, bmax, e_rows,
+                                     ws->max_grid, stream, &plan.grid);
+    } else {
+        void *params[] = {&a};
+        e = cudaLaunchKernel(plan.kernel, dim3(plan.grid), dim3(plan.block), params,
+                             plan.smem, stream);
+    }
     if (e != cudaSuccess) return cuda_fail(e, "fused sync launch");
     if (o.time_kernel && (e = cudaEventRecord(ws->ev1, stream)) != cudaSuccess)
         return cuda_fail(e, "cudaEventRecord");
@@ -521,7 +583,7 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
         return fail(ALOCO_ERR_CUDA,
                     "bulk-copy pipeline wait timed out; outputs are incomplete");
     }
-    finalize_stats(ws->host, nf, M, o.eps, st);
+    finalize_stats(ws->host, nf, M, o.eps, int8 ? 1.0 : 1.0 / ((double)M * (double)M), st);
     st->grid = plan.grid;
     st->pass_used = tma ? ALOCO_PASS_BULK_COPY : ALOCO_PASS_REGISTERS;
     if (o.time_kernel) {
@@ -535,6 +597,117 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
         return fail(ALOCO_ERR_NONFINITE,
                     "round produced %lld non-finite elements (D=%g, C=%g)",
                     (long long)st->nonfinite, st->D, st->C);
+    t_err.clear();
+    return ALOCO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int aloco_sync_ex(float *global, float *momentum, void *const *locals,
+                  size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                  int64_t H_base, int64_t step,
+                  const aloco_schedule_t *schedule, double outer_lr,
+                  double outer_beta, const aloco_opts_t *opts,
+                  aloco_stats_t *stats_out) {
+    return sync_impl(global, momentum, locals, N, M, dtype, H_sel, H_base, step,
+                     schedule, outer_lr, outer_beta, false, nullptr, 0, opts,
+                     stats_out);
+}
+
+int aloco_sync_int8(float *global, float *momentum, void *const *locals,
+                    size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                    int64_t H_base, int64_t step,
+                    const aloco_schedule_t *schedule, double outer_lr,
+                    double outer_beta, const int64_t *part_sizes, int n_parts,
+                    const aloco_opts_t *opts, aloco_stats_t *stats_out) {
+    return sync_impl(global, momentum, locals, N, M, dtype, H_sel, H_base, step,
+                     schedule, outer_lr, outer_beta, true, part_sizes, n_parts,
+                     opts, stats_out);
+}
+
+int64_t aloco_int8_num_blocks(const int64_t *part_sizes, int n_parts) {
+    if (!part_sizes || n_parts < 1) {
+        fail(ALOCO_ERR_ARG, "part_sizes is NULL or n_parts < 1");
+        return -1;
+    }
+    int64_t nb = 0;
+    for (int p = 0; p < n_parts; ++p) {
+        if (part_sizes[p] < 1) {
+            fail(ALOCO_ERR_ARG, "part %d has size %lld", p, (long long)part_sizes[p]);
+            return -1;
+        }
+        nb += (part_sizes[p] + 4095) / 4096;
+    }
+    return nb;
+}
+
+}  // extern "C"
+
+namespace {
+
+// Common set-up of the stand-alone codec calls.
+int codec_setup(size_t N, const int64_t *parts, int n_parts, aloco::Int8Parts *P,
+                int *sm_count) {
+    if (N == 0) return fail(ALOCO_ERR_ARG, "N must be >= 1");
+    int rc = build_parts(parts, n_parts, N, P);
+    if (rc != ALOCO_OK) return rc;
+    int device = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    e = cudaDeviceGetAttribute(sm_count, cudaDevAttrMultiProcessorCount, device);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    return ALOCO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int aloco_int8_encode(const float *x, size_t N, const int64_t *part_sizes,
+                      int n_parts, int8_t *codes, float *scales, float *decoded,
+                      void *stream) {
+    if (!x || !codes || !scales) return fail(ALOCO_ERR_ARG, "NULL buffer");
+    static thread_local aloco::Int8Parts P;
+    int sms = 0;
+    int rc = codec_setup(N, part_sizes, n_parts, &P, &sms);
+    if (rc != ALOCO_OK) return rc;
+    int device = 0;
+    cudaGetDevice(&device);
+    if ((rc = check_buffer(x, N * 4, device, "x")) != ALOCO_OK) return rc;
+    if ((rc = check_buffer(codes, N, device, "codes")) != ALOCO_OK) return rc;
+    if ((rc = check_buffer(scales, (size_t)P.blk[P.n_parts] * 4, device, "scales")) != ALOCO_OK)
+        return rc;
+    if (decoded && (rc = check_buffer(decoded, N * 4, device, "decoded")) != ALOCO_OK)
+        return rc;
+    const bool vec = (((uintptr_t)x | (uintptr_t)decoded) & 15) == 0 &&
+                     ((uintptr_t)codes & 3) == 0;
+    cudaError_t e = aloco::launch_int8_encode(x, codes, scales, decoded, vec, P, sms,
+                                              (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "int8 encode launch");
+    t_err.clear();
+    return ALOCO_OK;
+}
+
+int aloco_int8_decode(const int8_t *codes, const float *scales, size_t N,
+                      const int64_t *part_sizes, int n_parts, float *out,
+                      void *stream) {
+    if (!codes || !scales || !out) return fail(ALOCO_ERR_ARG, "NULL buffer");
+    static thread_local aloco::Int8Parts P;
+    int sms = 0;
+    int rc = codec_setup(N, part_sizes, n_parts, &P, &sms);
+    if (rc != ALOCO_OK) return rc;
+    int device = 0;
+    cudaGetDevice(&device);
+    if ((rc = check_buffer(codes, N, device, "codes")) != ALOCO_OK) return rc;
+    if ((rc = check_buffer(scales, (size_t)P.blk[P.n_parts] * 4, device, "scales")) != ALOCO_OK)
+        return rc;
+    if ((rc = check_buffer(out, N * 4, device, "out")) != ALOCO_OK) return rc;
+    const bool vec = ((uintptr_t)out & 15) == 0 && ((uintptr_t)codes & 3) == 0;
+    cudaError_t e = aloco::launch_int8_decode(codes, scales, out, vec, P, sms,
+                                              (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "int8 decode launch");
     t_err.clear();
     return ALOCO_OK;
 }
@@ -555,6 +728,9 @@ void aloco_shutdown(void) {
         if (ws->ev1) cudaEventDestroy(ws->ev1);
         if (ws->host) cudaFreeHost(ws->host);
         if (ws->dev) cudaFree(ws->dev);
+        if (ws->i8) cudaFree(ws->i8);
+        ws->i8 = nullptr;
+        ws->i8_cap = 0;
         ws->ev0 = ws->ev1 = nullptr;
         ws->host = nullptr;
         ws->dev = nullptr;

@@ -82,12 +82,38 @@ cudaError_t plan_sync_tma_bf16(int M, int64_t nvec, int sm_count,
 // requested aloco_pass.
 bool use_tma(int pass, int M, aloco_dtype dtype, int64_t nvec);
 
+// Tensor parts of an INT8-communicated round, passed by value to the
+// kernels: part p covers elements [off[p], off[p+1]) and its codec blocks
+// are blk[p] .. blk[p+1]-1.
+constexpr int kInt8MaxParts = 1024;
+struct Int8Parts {
+    int64_t off[kInt8MaxParts + 1];
+    int64_t blk[kInt8MaxParts + 1];
+    int n_parts;
+};
+
+// Enqueue the two passes of an INT8 round.  bmax holds nblocks * M
+// unsigned (per-block worker maxima, cleared here), e_rows max_grid * 16
+// doubles (device scratch).
+cudaError_t launch_int8_round(const SyncArgs &a, const Int8Parts &P,
+                              aloco_dtype dtype, int sm_count, unsigned *bmax,
+                              double *e_rows, int max_grid, cudaStream_t stream,
+                              int *grid_out);
+cudaError_t launch_int8_encode(const float *x, int8_t *codes, float *scales,
+                               float *decoded, bool vec_ok, const Int8Parts &P,
+                               int sm_count, cudaStream_t stream);
+cudaError_t launch_int8_decode(const int8_t *codes, const float *scales,
+                               float *out, bool vec_ok, const Int8Parts &P,
+                               int sm_count, cudaStream_t stream);
+
 // Host helpers shared by the entry points (aloco_host.cpp).
 int report_error(int code, const char *msg);
 int check_buffer(const void *p, size_t bytes, int device, const char *name);
 void fill_default_opts(aloco_opts_t *o);
 void split_coef(double x, float *hi, float *lo);
+// b_scale converts the last total into ||Dbar||^2: 1/M^2 when the pass
+// accumulated (sum_m Delta_m)^2, 1 when it accumulated the aggregate itself.
 void finalize_stats(const double *totals, unsigned long long nf, int M,
-                    double eps, aloco_stats_t *st);
+                    double eps, double b_scale, aloco_stats_t *st);
 
 }  // namespace aloco

@@ -237,7 +237,7 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
     if (perr != 0)
         return errf(ALOCO_ERR_CUDA,
                     "bulk-copy pipeline wait timed out; outputs are incomplete");
-    aloco::finalize_stats(host, nf, M, o.eps, st);
+    aloco::finalize_stats(host, nf, M, o.eps, 1.0 / ((double)M * (double)M), st);
     st->grid = plan.grid;
     st->pass_used = tma ? ALOCO_PASS_BULK_COPY : ALOCO_PASS_REGISTERS;
     if (st->nonfinite > 0 || !std::isfinite(st->D) || !std::isfinite(st->C))

@@ -1,0 +1,210 @@
+"""INT8 pseudo-gradient communication (App. G.1) on the GPU against the
+oracle: the codec bit for bit (codes, scales and decoded values decide
+integers in FP32 on both sides), and the INT8-communicated round."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2609_36662_gb300 import aloco as A
+from paper_2609_36662_gb300 import workloads as W
+
+from _parity import (assert_bf16_replica, assert_corr, assert_field,
+                     assert_stats, gpu_inputs, oracle_corr, schedule_pair,
+                     to_numpy_bits)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+PARTS = {
+    "one_part": None,
+    "ragged": [3 * 4096 + 64, 768, 5001, 12, 4096, 7],
+    "llama_like": [32000 * 64, 64, 64 * 64, 64 * 16, 64 * 16, 64 * 64, 64,
+                   64 * 172, 64 * 172, 172 * 64, 64],
+}
+
+
+def _vec(n, seed, kind="normal"):
+    rng = np.random.default_rng(seed)
+    y = rng.normal(0, 1e-3, n).astype(np.float32)
+    if kind == "special":
+        y[:4096] = 0.0                       # an all-zero block
+        y[5000] = np.float32(3e38)           # near the top of fp32
+        y[12288:16384] = np.float32(1e-42)   # a block of subnormals only
+        y[20000] = np.nan
+        y[30000] = np.inf
+    return y
+
+
+def _same_bits(a, b):
+    """Bit-identical fp32 values, except that any NaN matches any NaN (the
+    payload of a NaN produced by arithmetic differs between CPU and GPU)."""
+    na, nb = np.isnan(a), np.isnan(b)
+    np.testing.assert_array_equal(na, nb)
+    np.testing.assert_array_equal(a[~na].view(np.uint32),
+                                  b[~nb].view(np.uint32))
+
+
+@pytest.mark.parametrize("parts_name", sorted(PARTS))
+@pytest.mark.parametrize("kind", ["normal", "special"])
+def test_codec_bit_exact(parts_name, kind):
+    parts = PARTS[parts_name]
+    N = sum(parts) if parts else 3 * 4096 + 1000
+    if kind == "special" and N < 40000:
+        N = 40000 if parts is None else N
+    y = _vec(N, 3, kind if N >= 40000 else "normal")
+    codes, scales, dec = A.int8_encode(torch.from_numpy(y).cuda(), parts)
+    oc, osc, odec = O.int8_encode(y, parts)
+    np.testing.assert_array_equal(codes.cpu().numpy(), oc)
+    _same_bits(scales.cpu().numpy(), osc)
+    _same_bits(dec.cpu().numpy(), odec)
+    back = A.int8_decode(codes, scales, parts)
+    _same_bits(back.cpu().numpy(), odec)
+    assert A.int8_num_blocks(parts or [N]) == O.int8_blocks(parts or [N])
+
+
+def _int8_oracle(w, g, v, xs, parts, step, hsel):
+    corr = oracle_corr(w, step, hsel)
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+    return corr, O.int8_round(g.cpu().numpy(), v.cpu().numpy(),
+                              [to_numpy_bits(x) for x in xs], dt, parts,
+                              corr.mu_t, corr.eta_out, corr.inv_norm)
+
+
+def _compare(w, st, corr, orc, g, v, xs):
+    assert st["status"] == A.OK
+    assert_corr(st["corr"], corr)
+    assert_stats(st, orc, w.M)
+    assert_field(g.cpu().numpy(), orc["g"], "theta'")
+    assert_field(v.cpu().numpy(), orc["v"], "v'")
+    for m, x in enumerate(xs):
+        if w.dtype == "f32":
+            assert_field(x.cpu().numpy(), orc["x"][m], f"replica {m}")
+        else:
+            assert_bf16_replica(to_numpy_bits(x), orc["x"][m], orc["g"],
+                                f"replica {m}")
+
+
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+@pytest.mark.parametrize("M", [1, 2, 3, 8, 16])
+@pytest.mark.parametrize("parts_name", ["one_part", "ragged", "llama_like"])
+def test_int8_round_matches_oracle(dt, M, parts_name):
+    parts = PARTS[parts_name]
+    N = sum(parts) if parts else 5 * 4096 + 333
+    w = W.small(N, M, dt, seed=40 + M)
+    g, v, xs = gpu_inputs(w)
+    v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(M))
+    corr, orc = _int8_oracle(w, g, v, xs, parts, w.start_step, w.H_sel[0])
+    sa, _ = schedule_pair(w.schedule)
+    st = A.sync_int8(g, v, xs, parts=parts, H_sel=w.H_sel[0], H_base=w.H_base,
+                     step=w.start_step, schedule=sa, outer_lr=w.outer_lr,
+                     outer_beta=w.outer_beta)
+    _compare(w, st, corr, orc, g, v, xs)
+
+
+def test_int8_round_with_normalisation_and_nonfinite():
+    parts = PARTS["ragged"]
+    N = sum(parts)
+    w = W.small(N, 4, "f32", seed=50, H_sel=400)
+    g, v, xs = gpu_inputs(w)
+    xs[2][100] = float("nan")
+    sa, _ = schedule_pair(w.schedule)
+    corr = O.correction(O.Schedule(), w.start_step, 400, w.H_base, w.outer_lr,
+                        w.outer_beta, normalize=True)
+    orc = O.int8_round(g.cpu().numpy(), v.cpu().numpy(),
+                       [x.cpu().numpy() for x in xs], O.F32, parts,
+                       corr.mu_t, corr.eta_out, corr.inv_norm)
+    st = A.sync_int8(g, v, xs, parts=parts, H_sel=400, H_base=w.H_base,
+                     step=w.start_step, schedule=sa, outer_lr=w.outer_lr,
+                     outer_beta=w.outer_beta,
+                     opts=A.default_opts(normalize=1))
+    assert st["status"] == A.ERR_NONFINITE
+    assert st["nonfinite"] == orc["nonfinite"] > 0
+    finite = np.isfinite(orc["g"])
+    assert_field(g.cpu().numpy()[finite], orc["g"][finite], "theta'")
+
+
+def test_int8_round_full_size_llama150m():
+    """The 150M layout (111 tensor parts, 8 fp32 workers) in one INT8 round:
+    sampled whole codec blocks against the oracle, and the full statistics
+    from the oracle over every part (threaded over parts)."""
+    import concurrent.futures as cf
+    w = W.llama_150m()
+    parts = W.tensor_sizes(w)
+    g, v, xs = gpu_inputs(w)
+    g_in, v_in = g.clone(), v.clone()
+    x_in = [x.clone() for x in xs]
+    step, hsel = W.steps_of_rounds(w)[0]
+    corr = oracle_corr(w, step, hsel)
+    sa, _ = schedule_pair(w.schedule)
+    st = A.sync_int8(g, v, xs, parts=parts, H_sel=hsel, H_base=w.H_base,
+                     step=step, schedule=sa, outer_lr=w.outer_lr,
+                     outer_beta=w.outer_beta)
+    assert st["status"] == A.OK
+    assert_corr(st["corr"], corr)
+    offs = np.concatenate([[0], np.cumsum(parts)])
+    # full statistics: the oracle over each part on its own thread
+    E = np.zeros((len(parts), w.M))
+    B = np.zeros(len(parts))
+
+    def work(p):
+        s, e = int(offs[p]), int(offs[p + 1])
+        r = O.int8_round(g_in[s:e].cpu().numpy(), v_in[s:e].cpu().numpy(),
+                         [x[s:e].cpu().numpy() for x in x_in], O.F32,
+                         [e - s], corr.mu_t, corr.eta_out, corr.inv_norm)
+        E[p] = r["drift"]
+        B[p] = r["mean_sq_norm"]
+        return p, s, r
+    rng = np.random.default_rng(0)
+    check = set(rng.choice(len(parts), 12, replace=False).tolist()) | {0, 1,
+                                                                      len(parts) - 1}
+    with cf.ThreadPoolExecutor(16) as ex:
+        for p, s, r in ex.map(work, range(len(parts))):
+            if p in check:
+                e = s + r["g"].size
+                assert_field(g[s:e].cpu().numpy(), r["g"], f"theta' part {p}")
+                assert_field(v[s:e].cpu().numpy(), r["v"], f"v' part {p}")
+    Em = [float(E[:, m].sum()) for m in range(w.M)]
+    D = sum(Em) / w.M
+    Bt = float(B.sum())
+    orc = {"D": D, "C": w.M * Bt / (D + 1e-8), "mean_sq_norm": Bt,
+           "drift": Em}
+    assert_stats(st, orc, w.M)
+
+
+def test_codec_decisions_at_rounding_ties():
+    """The GPU divides by the block scale with a correctly rounded reciprocal
+    and two exact-residual corrections; the oracle uses IEEE division.  Put
+    values on, and one ulp either side of, half-integer multiples of the
+    scale in 4096 blocks with scales spread over 2^-60 .. 2^60, plus random
+    values: every code must agree."""
+    rng = np.random.default_rng(123)
+    nb = 4096
+    y = np.empty(nb * 4096, np.float32)
+    for b in range(nb):
+        s_target = np.float32(2.0 ** rng.uniform(-60, 60))
+        amax = np.float32(s_target * 127)
+        blk = np.empty(4096, np.float32)
+        blk[0] = amax                                   # fixes the scale
+        s = np.float32(amax / np.float32(127))
+        k = rng.integers(-126, 126, 4095)
+        half = ((k + 0.5) * s.astype(np.float64)).astype(np.float32)
+        which = rng.integers(0, 4, 4095)
+        blk[1:] = np.where(which == 0, half,
+                  np.where(which == 1, np.nextafter(half, np.float32(np.inf)),
+                  np.where(which == 2, np.nextafter(half, np.float32(-np.inf)),
+                           (rng.uniform(-127, 127, 4095) * s).astype(np.float32))))
+        y[b * 4096:(b + 1) * 4096] = blk
+    codes, scales, _ = A.int8_encode(torch.from_numpy(y).cuda())
+    oc, osc, _ = O.int8_encode(y)
+    np.testing.assert_array_equal(scales.cpu().numpy().view(np.uint32),
+                                  osc.view(np.uint32))
+    np.testing.assert_array_equal(codes.cpu().numpy(), oc)
