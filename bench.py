@@ -42,7 +42,8 @@ METRIC = ("outer-sync rounds/s and achieved HBM GB/s (fraction of GB300 "
 UNIT = "rounds/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-PASSES = {"auto": 0, "registers": 1, "bulk_copy": 2}
+PASSES = {"auto": 0, "registers": 1, "bulk_copy": 2, "int8_split": 3,
+          "int8_fused": 4}
 
 
 def workloads_by_name():
@@ -77,13 +78,27 @@ def hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash() -> str:
+# the sources each timed kernel is compiled from; a recorded ncu traffic
+# figure stays valid only while these files are unchanged
+KERNEL_SOURCES = {
+    "sync_kernel": ("aloco_internal.h", "aloco_sync_kernel.cuh",
+                    "aloco_sync_f32.cu", "aloco_sync_bf16.cu"),
+    "sync_tma_kernel": ("aloco_internal.h", "aloco_sync_kernel.cuh",
+                        "aloco_sync_tma.cuh", "aloco_sync_tma_f32.cu",
+                        "aloco_sync_tma_bf16.cu"),
+    "int8_split_kernels": ("aloco_internal.h", "aloco_sync_kernel.cuh",
+                           "aloco_int8.cuh", "aloco_int8.cu"),
+    "int8_fused_kernel": ("aloco_internal.h", "aloco_sync_kernel.cuh",
+                          "aloco_int8.cuh", "aloco_int8_fused.cu"),
+}
+
+
+def kernel_source_hash(kernel: str) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_36662_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(f.read())
+    for name in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read())
     return h.hexdigest()[:16]
 
 
@@ -97,7 +112,7 @@ def recorded_traffic(workload: str, kernel: str):
     except Exception:
         return None
     entry = rec.get(f"{workload}/{kernel}")
-    if not entry or entry.get("kernel_hash") != kernel_source_hash():
+    if not entry or entry.get("kernel_hash") != kernel_source_hash(kernel):
         return None
     return entry.get("dram_bytes_per_launch")
 
@@ -191,9 +206,24 @@ def job_value(units_per_rank: float, seconds_max: float, world: int) -> float:
 
 # ------------------------------------------------------------ CPU oracle
 
-def oracle_sample(w, g, v, xs, elems: int, step: int, H_sel: int):
+def prefix_parts(parts, n: int):
+    """The tensor parts of the first n elements (the last one cut short)."""
+    out, acc = [], 0
+    for p in parts:
+        if acc >= n:
+            break
+        take = min(p, n - acc)
+        out.append(take)
+        acc += take
+    return out
+
+
+def oracle_sample(w, g, v, xs, elems: int, step: int, H_sel: int,
+                  comm: str = "fp32"):
     """Time the oracle (single thread, as it stands) on the first `elems`
-    elements of the round.  Returns seconds."""
+    elements of the round (the INT8-communicated round when comm is
+    "int8", with the codec's blocks cut at the same tensor boundaries).
+    Returns seconds."""
     import numpy as np
     import torch
     import oracle as O
@@ -208,16 +238,24 @@ def oracle_sample(w, g, v, xs, elems: int, step: int, H_sel: int):
     s = w.schedule
     sched = O.Schedule(s.kind, s.peak_lr, s.final_lr, s.warmup_steps,
                        s.total_steps)
+    dt = O.F32 if w.dtype == "f32" else O.BF16
     t0 = time.perf_counter()
-    O.sync_round(gh, vh, xh, O.F32 if w.dtype == "f32" else O.BF16, sched,
-                 step, H_sel, w.H_base, w.outer_lr, w.outer_beta)
+    if comm == "int8":
+        from paper_2609_36662_gb300 import workloads as W
+        corr = O.correction(sched, step, H_sel, w.H_base, w.outer_lr,
+                            w.outer_beta)
+        O.int8_round(gh, vh, xh, dt, prefix_parts(W.tensor_sizes(w), n),
+                     corr.mu_t, corr.eta_out, corr.inv_norm)
+    else:
+        O.sync_round(gh, vh, xh, dt, sched, step, H_sel, w.H_base,
+                     w.outer_lr, w.outer_beta)
     return time.perf_counter() - t0, n
 
 
-def calibrated_sample(w, g, v, xs, step, H_sel, target_s):
+def calibrated_sample(w, g, v, xs, step, H_sel, target_s, comm="fp32"):
     """Pick a sample size whose oracle run takes about target_s seconds."""
     probe = min(w.numel, 1 << 20)
-    t, n = oracle_sample(w, g, v, xs, probe, step, H_sel)
+    t, n = oracle_sample(w, g, v, xs, probe, step, H_sel, comm)
     per_elem = t / n
     want = int(target_s / max(per_elem, 1e-12))
     want = max(1 << 16, min(w.numel, want))
@@ -247,13 +285,14 @@ def run_reference(args, w):
 
     # calibrate on the first chunk, then draw only the chunks the sample needs
     xs = endpoints(1)
-    sample = calibrated_sample(w, g, v, xs, step0, h0, args.ref_step_seconds)
+    sample = calibrated_sample(w, g, v, xs, step0, h0, args.ref_step_seconds,
+                               args.comm)
     need = (sample + W.CHUNK - 1) // W.CHUNK
     if need > 1:
         xs = endpoints(need)
     times = []
     for k, (step, hsel) in enumerate(rounds):
-        t, n = oracle_sample(w, g, v, xs, sample, step, hsel)
+        t, n = oracle_sample(w, g, v, xs, sample, step, hsel, args.comm)
         if k >= args.warmup:
             times.append(t)
     sec_per_round = statistics.mean(times) * w.numel / sample
@@ -264,7 +303,7 @@ def run_reference(args, w):
         "ms_per_step": sec_per_round * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": config_block(w),
+        "config": dict(config_block(w), comm=args.comm),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1,
                          "kind": "oracle",
                          "sample": f"first {sample} of {w.numel} parameters "
@@ -320,8 +359,9 @@ def run_cuda(args, w):
     cpu_baseline = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         step0, h0 = rounds[0]
-        sample = calibrated_sample(w, g, v, xs, step0, h0, args.cpu_seconds)
-        t, n = oracle_sample(w, g, v, xs, sample, step0, h0)
+        sample = calibrated_sample(w, g, v, xs, step0, h0, args.cpu_seconds,
+                                   args.comm)
+        t, n = oracle_sample(w, g, v, xs, sample, step0, h0, args.comm)
         cpu_baseline = {"value": (n / w.numel) / t, "unit": UNIT, "cores": 1,
                         "kind": "oracle",
                         "sample": f"first {n} of {w.numel} parameters x "
@@ -374,9 +414,9 @@ def run_cuda(args, w):
     for k in range(args.warmup, args.warmup + args.steps):
         step_ms.append(ev[k][0].elapsed_time(ev[k][1]))
 
-    kernel_name = ("int8_round_kernel" if args.comm == "int8" else
-                   "sync_tma_kernel" if st_first.get("pass_used") == 2
-                   else "sync_kernel")
+    kernel_name = {2: "sync_tma_kernel", 3: "int8_split_kernels",
+                   4: "int8_fused_kernel"}.get(st_first.get("pass_used"),
+                                               "sync_kernel")
     ms_step = statistics.mean(step_ms)
     ms_step = reduce_max(ms_step, world, device)
     ms_kern = reduce_max(statistics.mean(kern_ms), world, device)
@@ -387,8 +427,9 @@ def run_cuda(args, w):
     # end to end through the C ABI with host buffers: H2D of the round's
     # inputs from pinned memory, the round, D2H of theta' and v'
     e2e = None
-    if not args.no_e2e and args.comm == "fp32":
-        e2e = run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device)
+    if not args.no_e2e:
+        e2e = run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
+                      parts if args.comm == "int8" else None)
 
     if rank == 0:
         line = {
@@ -412,7 +453,9 @@ def run_cuda(args, w):
                          "algorithmic_bytes_per_launch": w.bytes_per_round()},
             "cpu_baseline": cpu_baseline,
             "e2e": e2e,
-            "gpu_launches": args.steps,
+            # the split INT8 round is two kernels (block scales, then apply)
+            "gpu_launches": args.steps * (2 if kernel_name == "int8_split_kernels"
+                                          else 1),
             "clocks": clocks.summary(),
             "status_ok": all(s_ in (A.OK,) for s_ in statuses),
             "wall_s_timed_loop": t_wall,
@@ -423,7 +466,8 @@ def run_cuda(args, w):
     return 0
 
 
-def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device):
+def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
+            int8_parts=None):
     import torch
     from paper_2609_36662_gb300 import aloco as A
     from paper_2609_36662_gb300 import workloads as W
@@ -461,9 +505,15 @@ def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device):
             v.copy_(hv, non_blocking=True)
             for a, b in zip(xs, hx):
                 a.copy_(b, non_blocking=True)
-            A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step,
-                   schedule=sched, outer_lr=w.outer_lr,
-                   outer_beta=w.outer_beta, stream=stream)
+            if int8_parts is not None:
+                A.sync_int8(g, v, xs, parts=int8_parts, H_sel=hsel,
+                            H_base=w.H_base, step=step, schedule=sched,
+                            outer_lr=w.outer_lr, outer_beta=w.outer_beta,
+                            stream=stream)
+            else:
+                A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step,
+                       schedule=sched, outer_lr=w.outer_lr,
+                       outer_beta=w.outer_beta, stream=stream)
             og.copy_(g, non_blocking=True)
             ov.copy_(v, non_blocking=True)
             e1.record(stream)

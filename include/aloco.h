@@ -114,11 +114,22 @@ typedef enum {
  *              consumer warps compute from shared memory (M <= 16, 16-byte
  *              aligned buffers; otherwise REGISTERS runs);
  *   AUTO       the faster of the two as measured on GB300: at present the
- *              register-streaming pass for every (M, dtype). */
+ *              register-streaming pass for every (M, dtype).
+ * The INT8-communicated round (aloco_sync_int8) has two forms of its own:
+ *   INT8_SPLIT a block-scale kernel, then an apply kernel that reads the
+ *              replicas again (any M <= 16);
+ *   INT8_FUSED one kernel whose threads hold their replica values in
+ *              registers, reading every replica once (bf16 M <= 8, fp32
+ *              M <= 4; ALOCO_ERR_ARG otherwise);
+ *   AUTO       the form measured faster on GB300 for (M, dtype).
+ * aloco_sync / aloco_sync_ex reject the INT8 values and aloco_sync_int8 the
+ * REGISTERS / BULK_COPY values with ALOCO_ERR_ARG. */
 typedef enum {
     ALOCO_PASS_AUTO = 0,
     ALOCO_PASS_REGISTERS = 1,
-    ALOCO_PASS_BULK_COPY = 2
+    ALOCO_PASS_BULK_COPY = 2,
+    ALOCO_PASS_INT8_SPLIT = 3,
+    ALOCO_PASS_INT8_FUSED = 4
 } aloco_pass;
 
 /* Options.  aloco_default_opts() fills the paper's settings

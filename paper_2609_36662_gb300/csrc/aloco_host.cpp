@@ -110,7 +110,7 @@ int correction_impl(const aloco_schedule_t *sched, int64_t step,
     if (!std::isfinite(outer_lr)) return fail(ALOCO_ERR_ARG, "outer_lr must be finite");
     if (o.blocks_per_sm < 0)
         return fail(ALOCO_ERR_ARG, "blocks_per_sm must be >= 0");
-    if (o.pass < ALOCO_PASS_AUTO || o.pass > ALOCO_PASS_BULK_COPY)
+    if (o.pass < ALOCO_PASS_AUTO || o.pass > ALOCO_PASS_INT8_FUSED)
         return fail(ALOCO_ERR_ARG, "unknown pass %d", o.pass);
     if (o.mode != ALOCO_CORR_FULL && o.mode != ALOCO_CORR_MOMENTUM_ONLY &&
         o.mode != ALOCO_CORR_NONE)
@@ -261,6 +261,13 @@ GetAddressRangeFn address_range_fn() {
 // Helpers with external linkage: also used by the allocation-free entry
 // point (aloco_noalloc.cu).
 namespace aloco {
+
+bool use_int8_fused(int pass, int M, aloco_dtype dtype) {
+    if (!int8_fused_fits(M, dtype)) return false;
+    if (pass == ALOCO_PASS_INT8_FUSED) return true;
+    if (pass == ALOCO_PASS_INT8_SPLIT) return false;
+    return true;  // AUTO
+}
 
 bool use_tma(int pass, int M, aloco_dtype dtype, int64_t nvec) {
     if (M < 1 || M > 16 || nvec < kTmaTilePacks) return false;
@@ -429,6 +436,12 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
                     int8 ? 16 : ALOCO_MAX_WORKERS);
     if (dtype != ALOCO_F32 && dtype != ALOCO_BF16)
         return fail(ALOCO_ERR_ARG, "unknown replica dtype %d", (int)dtype);
+    const bool int8_pass = o.pass == ALOCO_PASS_INT8_SPLIT || o.pass == ALOCO_PASS_INT8_FUSED;
+    if (int8 ? (o.pass == ALOCO_PASS_REGISTERS || o.pass == ALOCO_PASS_BULK_COPY)
+             : int8_pass)
+        return fail(ALOCO_ERR_ARG, "pass %d does not apply to this round", o.pass);
+    if (int8 && o.pass == ALOCO_PASS_INT8_FUSED && !aloco::int8_fused_fits(M, dtype))
+        return fail(ALOCO_ERR_ARG, "the fused INT8 round takes bf16 M <= 8 or fp32 M <= 4");
     if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
     if (N > 0 && (!global || !momentum || !locals))
         return fail(ALOCO_ERR_ARG, "NULL buffer");
@@ -514,7 +527,12 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     const int64_t work = a.nvec > 0 ? a.nvec : a.n;
     aloco::LaunchPlan plan;
     const bool tma = !int8 && aloco::use_tma(o.pass, M, dtype, a.nvec);
-    if (int8) {
+    const bool fused = int8 && aloco::use_int8_fused(o.pass, M, dtype);
+    if (fused) {
+        plan.grid = 0;
+        plan.block = 0;
+        plan.kernel = nullptr;
+    } else if (int8) {
         // scratch of the two INT8 passes: per-block worker scales and the
         // per-CTA drift energies of pass 1 (grown on demand, kept cached)
         const size_t need = (size_t)P.blk[P.n_parts] * M * sizeof(float) + 256 +
@@ -552,7 +570,10 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     cudaStream_t stream = (cudaStream_t)o.stream;
     if (o.time_kernel && (e = cudaEventRecord(ws->ev0, stream)) != cudaSuccess)
         return cuda_fail(e, "cudaEventRecord");
-    if (int8) {
+    if (fused) {
+        e = aloco::launch_int8_fused(a, P, dtype, ws->sm_count, ws->max_grid, stream,
+                                     &plan.grid);
+    } else if (int8) {
         double *e_rows = reinterpret_cast<double *>(ws->i8);
         unsigned *bmax = reinterpret_cast<unsigned *>(
             ws->i8 + (size_t)ws->max_grid * 16 * sizeof(double));
@@ -585,7 +606,10 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     }
     finalize_stats(ws->host, nf, M, o.eps, int8 ? 1.0 : 1.0 / ((double)M * (double)M), st);
     st->grid = plan.grid;
-    st->pass_used = tma ? ALOCO_PASS_BULK_COPY : ALOCO_PASS_REGISTERS;
+    st->pass_used = fused ? ALOCO_PASS_INT8_FUSED
+                    : int8 ? ALOCO_PASS_INT8_SPLIT
+                    : tma  ? ALOCO_PASS_BULK_COPY
+                           : ALOCO_PASS_REGISTERS;
     if (o.time_kernel) {
         float ms = -1.f;
         if (cudaEventElapsedTime(&ms, ws->ev0, ws->ev1) == cudaSuccess)

@@ -81,6 +81,8 @@ cudaError_t plan_sync_tma_bf16(int M, int64_t nvec, int sm_count,
 // Whether a round of M workers (dtype) uses the bulk-copy pass, given the
 // requested aloco_pass.
 bool use_tma(int pass, int M, aloco_dtype dtype, int64_t nvec);
+// Whether an INT8 round of M workers (dtype) uses the fused form.
+bool use_int8_fused(int pass, int M, aloco_dtype dtype);
 
 // Tensor parts of an INT8-communicated round, passed by value to the
 // kernels: part p covers elements [off[p], off[p+1]) and its codec blocks
@@ -92,13 +94,19 @@ struct Int8Parts {
     int n_parts;
 };
 
-// Enqueue the two passes of an INT8 round.  bmax holds nblocks * M
-// unsigned (per-block worker maxima, cleared here), e_rows max_grid * 16
-// doubles (device scratch).
+// Enqueue the split form of an INT8 round (two kernels).  bmax holds
+// nblocks * M unsigned (per-block worker maxima, cleared here), e_rows
+// max_grid * 16 doubles (device scratch).
 cudaError_t launch_int8_round(const SyncArgs &a, const Int8Parts &P,
                               aloco_dtype dtype, int sm_count, unsigned *bmax,
                               double *e_rows, int max_grid, cudaStream_t stream,
                               int *grid_out);
+// The fused form (one kernel, no scratch beyond the reduction's): only
+// where int8_fused_fits(M, dtype), i.e. bf16 M <= 8 or fp32 M <= 4.
+bool int8_fused_fits(int M, aloco_dtype dtype);
+cudaError_t launch_int8_fused(const SyncArgs &a, const Int8Parts &P,
+                              aloco_dtype dtype, int sm_count, int max_grid,
+                              cudaStream_t stream, int *grid_out);
 cudaError_t launch_int8_encode(const float *x, int8_t *codes, float *scales,
                                float *decoded, bool vec_ok, const Int8Parts &P,
                                int sm_count, cudaStream_t stream);

@@ -211,6 +211,43 @@ def test_sync_argument_errors_before_any_device_work(lib):
     assert rc == A.ERR_ARG
 
 
+def test_pass_values_are_checked_against_the_round(lib):
+    """The INT8 forms are rejected by the plain round (and its allocation-free
+    entry point), the plain round's passes by the INT8 round, and the fused
+    INT8 form where its worker count does not fit; all before any device
+    work."""
+    import ctypes
+    s = A.Schedule.make()
+    base = 1 << 40
+    xs = [base + (k + 2) * (1 << 22) for k in range(2)]
+    for p in (A.PASS_INT8_SPLIT, A.PASS_INT8_FUSED, 5, -1):
+        for noalloc in (False, True):
+            rc, _ = A.sync_ptrs(base, base + (1 << 22), xs, 1000, A.F32, 150,
+                                100, 4000, s, 0.7, 0.9,
+                                opts=A.default_opts(pass_=p), noalloc=noalloc,
+                                raise_on_error=False)
+            assert rc == A.ERR_ARG, (p, noalloc)
+            assert "pass" in A.last_error()
+
+    def int8(M, dtype, p):
+        ptrs = (ctypes.c_void_p * M)(*[base + (k + 2) * (1 << 22)
+                                       for k in range(M)])
+        st = A.Stats()
+        return lib.aloco_sync_int8(base, base + (1 << 22), ptrs, 1000, M,
+                                   dtype, 150, 100, 4000, ctypes.byref(s),
+                                   0.7, 0.9, None, 0,
+                                   ctypes.byref(A.default_opts(pass_=p)),
+                                   ctypes.byref(st))
+    for p in (A.PASS_REGISTERS, A.PASS_BULK_COPY):
+        assert int8(2, A.F32, p) == A.ERR_ARG
+    assert int8(5, A.F32, A.PASS_INT8_FUSED) == A.ERR_ARG
+    assert int8(9, A.BF16, A.PASS_INT8_FUSED) == A.ERR_ARG
+    assert "fused" in A.last_error()
+    # accepted combinations get past argument checks (no device here)
+    assert int8(4, A.F32, A.PASS_INT8_FUSED) in (A.ERR_CUDA, A.ERR_ARG)
+    assert "fused" not in A.last_error()
+
+
 def test_empty_round_needs_no_device(lib):
     """N = 0 is a valid round: no kernel runs, the statistics are zero and
     the correction context is still reported."""

@@ -93,10 +93,20 @@ def _compare(w, st, corr, orc, g, v, xs):
                                 f"replica {m}")
 
 
+def _fits_fused(dt, M):
+    return M <= (8 if dt == "bf16" else 4)
+
+
+FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
+
+
+@pytest.mark.parametrize("form", sorted(FORMS))
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
-@pytest.mark.parametrize("M", [1, 2, 3, 8, 16])
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 16])
 @pytest.mark.parametrize("parts_name", ["one_part", "ragged", "llama_like"])
-def test_int8_round_matches_oracle(dt, M, parts_name):
+def test_int8_round_matches_oracle(dt, M, parts_name, form):
+    if form == "fused" and not _fits_fused(dt, M):
+        pytest.skip("the fused form holds bf16 M <= 8, fp32 M <= 4")
     parts = PARTS[parts_name]
     N = sum(parts) if parts else 5 * 4096 + 333
     w = W.small(N, M, dt, seed=40 + M)
@@ -106,8 +116,53 @@ def test_int8_round_matches_oracle(dt, M, parts_name):
     sa, _ = schedule_pair(w.schedule)
     st = A.sync_int8(g, v, xs, parts=parts, H_sel=w.H_sel[0], H_base=w.H_base,
                      step=w.start_step, schedule=sa, outer_lr=w.outer_lr,
-                     outer_beta=w.outer_beta)
+                     outer_beta=w.outer_beta,
+                     opts=A.default_opts(pass_=FORMS[form]))
+    assert st["pass_used"] == FORMS[form]
     _compare(w, st, corr, orc, g, v, xs)
+
+
+@pytest.mark.parametrize("dt,M", [("f32", 1), ("f32", 4), ("bf16", 2),
+                                  ("bf16", 5), ("bf16", 8)])
+def test_int8_forms_agree_bit_for_bit(dt, M):
+    """The fused and the split form take the same decisions in the same
+    arithmetic: theta', v' and the replicas are bit-identical; the
+    statistics differ at most by the order of their fp64 sums."""
+    parts = PARTS["llama_like"]
+    w = W.small(sum(parts), M, dt, seed=70 + M)
+    sa, _ = schedule_pair(w.schedule)
+    out = {}
+    for form, p in FORMS.items():
+        g, v, xs = gpu_inputs(w)
+        v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(M))
+        st = A.sync_int8(g, v, xs, parts=parts, H_sel=w.H_sel[0],
+                         H_base=w.H_base, step=w.start_step, schedule=sa,
+                         outer_lr=w.outer_lr, outer_beta=w.outer_beta,
+                         opts=A.default_opts(pass_=p))
+        out[form] = (st, g, v, xs)
+    (s1, g1, v1, x1), (s2, g2, v2, x2) = out["fused"], out["split"]
+    assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
+    assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))
+    for a, b in zip(x1, x2):
+        assert torch.equal(a, b)
+    for key in ("D", "C", "mean_sq_norm"):
+        assert s1[key] == pytest.approx(s2[key], rel=1e-12), key
+    assert s1["nonfinite"] == s2["nonfinite"] == 0
+
+
+def test_int8_auto_form():
+    """AUTO takes the fused form wherever it fits, the split form beyond."""
+    for dt, M, want in (("bf16", 8, A.PASS_INT8_FUSED),
+                        ("bf16", 9, A.PASS_INT8_SPLIT),
+                        ("f32", 4, A.PASS_INT8_FUSED),
+                        ("f32", 5, A.PASS_INT8_SPLIT)):
+        w = W.small(3 * 4096 + 5, M, dt, seed=3)
+        g, v, xs = gpu_inputs(w)
+        sa, _ = schedule_pair(w.schedule)
+        st = A.sync_int8(g, v, xs, H_sel=w.H_sel[0], H_base=w.H_base,
+                         step=w.start_step, schedule=sa, outer_lr=w.outer_lr,
+                         outer_beta=w.outer_beta)
+        assert st["pass_used"] == want, (dt, M)
 
 
 def test_int8_round_with_normalisation_and_nonfinite():
