@@ -81,15 +81,14 @@ def hbm_peak():
 # the sources each timed kernel is compiled from; a recorded ncu traffic
 # figure stays valid only while these files are unchanged
 KERNEL_SOURCES = {
-    "sync_kernel": ("aloco_internal.h", "aloco_sync_kernel.cuh",
-                    "aloco_sync_f32.cu", "aloco_sync_bf16.cu"),
-    "sync_tma_kernel": ("aloco_internal.h", "aloco_sync_kernel.cuh",
-                        "aloco_sync_tma.cuh", "aloco_sync_tma_f32.cu",
-                        "aloco_sync_tma_bf16.cu"),
-    "int8_split_kernels": ("aloco_internal.h", "aloco_sync_kernel.cuh",
-                           "aloco_int8.cuh", "aloco_int8.cu"),
-    "int8_fused_kernel": ("aloco_internal.h", "aloco_sync_kernel.cuh",
-                          "aloco_int8.cuh", "aloco_int8_fused.cu"),
+    "sync_kernel": ("aloco_sync_kernel.cuh", "aloco_sync_f32.cu",
+                    "aloco_sync_bf16.cu"),
+    "sync_tma_kernel": ("aloco_sync_kernel.cuh", "aloco_sync_tma.cuh",
+                        "aloco_sync_tma_f32.cu", "aloco_sync_tma_bf16.cu"),
+    "int8_split_kernels": ("aloco_sync_kernel.cuh", "aloco_int8.cuh",
+                           "aloco_int8.cu"),
+    "int8_fused_kernel": ("aloco_sync_kernel.cuh", "aloco_int8.cuh",
+                          "aloco_int8_fused.cu"),
 }
 
 

@@ -218,6 +218,20 @@ __device__ __forceinline__ int codec_code(float y, float s) {
     return (int)codec_code_f(y, s, __frcp_rn(s));
 }
 
+// Nearest integer, ties to even, of |t| < 2^22 on the fp32 adder: t + 1.5 *
+// 2^23 has no fraction bits left, so the addition rounds t at the units
+// place (to even on a tie), and subtracting the constant back is exact.
+// This keeps the hot loops off the conversion instruction, which on this
+// part issues at the low fp64 rate.  Explicit .rn PTX keeps the compiler
+// from folding the pair away.  (A zero result is +0.)
+constexpr float kRoundMagic = 12582912.f;  // 1.5 * 2^23
+__device__ __forceinline__ float rint_small(float t) {
+    float u, n;
+    asm("add.rn.f32 %0, %1, %2;" : "=f"(u) : "f"(t), "f"(kRoundMagic));
+    asm("add.rn.f32 %0, %1, %2;" : "=f"(n) : "f"(u), "f"(-kRoundMagic));
+    return n;
+}
+
 // The same code from the product y r alone when that is provably the same
 // decision: |y r - y/s| <= 2^-23 |y/s| < 2^-16 for |y r| < 127, so a
 // product at least 2^-14 away from every half-integer rounds like the
@@ -225,7 +239,7 @@ __device__ __forceinline__ int codec_code(float y, float s) {
 // finite take the exact quotient.
 __device__ __forceinline__ float codec_code_fast(float y, float s, float r) {
     const float t = __fmul_rn(y, r);
-    const float n = rintf(t);
+    const float n = rint_small(t);  // NaN or infinite t fails the test below
     if (fabsf(t) < 127.f && 0.5f - fabsf(t - n) > 0x1p-14f) return n;
     return codec_code_f(y, s, r);
 }
@@ -237,13 +251,24 @@ __device__ __forceinline__ float2 sub2(float2 a, float2 b) {  // RN(a - b)
     return __ffma2_rn(b, make_float2(-1.f, -1.f), a);
 }
 __device__ __forceinline__ float2 splat2(float a) { return make_float2(a, a); }
-// Paired product with explicit .rn rounding in PTX.  ptxas (CUDA 13.0) was
-// measured to contract a single-use paired product into a following paired
-// .rn add (a paired FMA), which skips the rounding of the decoded value q * s
-// that the codec defines; a one-ulp change in the mean then moves some
-// quotients across a half-integer.  So decoded values are summed with the
-// scalar __fadd_rn, which is never contracted, and the paired form serves
-// only products that are not added.
+// Paired sum and product with explicit .rn rounding in PTX.  ptxas (CUDA
+// 13.0) was measured to contract a single-use paired product into a
+// following paired .rn add (a paired FMA), which skips the rounding of the
+// decoded value q * s that the codec defines; a one-ulp change in the mean
+// then moves some quotients across a half-integer.  So decoded values are
+// summed with the scalar __fadd_rn, which is never contracted.  The paired
+// add serves only the rounding of a product in code2_fast, where a
+// contraction would round the exact product instead, and the half-integer
+// margin test there covers that difference.
+__device__ __forceinline__ float2 add2_rn(float2 a, float2 b) {
+    float2 r;
+    asm("{\n\t.reg .b64 pa, pb, pd;\n\t"
+        "mov.b64 pa, {%2, %3};\n\tmov.b64 pb, {%4, %5};\n\t"
+        "add.rn.f32x2 pd, pa, pb;\n\tmov.b64 {%0, %1}, pd;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
 __device__ __forceinline__ float2 mul2_rn(float2 a, float2 b) {
     float2 r;
     asm("{\n\t.reg .b64 pa, pb, pd;\n\t"
@@ -266,7 +291,9 @@ constexpr float kCodeMargin = 0.5f - 0x1p-14f;
 // and fl32(y/s) within 2^-17), and infinite or NaN products fail the test.
 __device__ __forceinline__ float2 code2_fast(float2 y, float r, bool &ok) {
     const float2 t = mul2_rn(y, splat2(r));
-    const float2 n = make_float2(rintf(t.x), rintf(t.y));
+    // rint_small of both lanes; an infinite or NaN product gives a NaN
+    // difference below and fails the test
+    const float2 n = add2_rn(add2_rn(t, splat2(kRoundMagic)), splat2(-kRoundMagic));
     const float2 d = sub2(t, n);  // exact: |t - n| <= 1/2
     ok = ok && fabsf(d.x) < kCodeMargin && fabsf(d.y) < kCodeMargin;
     return n;

@@ -258,3 +258,19 @@ def test_empty_round_needs_no_device(lib):
     assert d["D"] == 0.0 and d["C"] == 0.0 and d["nonfinite"] == 0
     oc = O.correction(O.Schedule(), 4000, 150, 100, 0.7, 0.9)
     assert d["corr"]["rho"] == pytest.approx(oc.rho, rel=1e-12)
+
+
+def test_int8_block_count_gives_the_papers_payload(lib):
+    """Host-only block count of the library (aloco_int8_num_blocks): the
+    Llama-3.1-8B parameter set moves 8.038 GB per INT8 synchronisation
+    (App. G.1; one byte per element plus one FP32 scale per block), the
+    same count as the oracle's; bad part lists are rejected."""
+    from paper_2609_36662_gb300 import workloads as W
+    parts = [n for _, n, _ in W.LLAMA31_8B.tensors()]
+    nb = A.int8_num_blocks(parts)
+    assert nb == O.int8_blocks(parts)
+    assert round((sum(parts) + 4 * nb) / 1e9, 3) == 8.038
+    assert A.int8_num_blocks([4096, 1, 4097]) == 1 + 1 + 2
+    for bad in ([0], [5, -1]):
+        with pytest.raises(A.AlocoError):
+            A.int8_num_blocks(bad)
