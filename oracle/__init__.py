@@ -81,6 +81,10 @@ def _load():
     lib.orc_int8_round.restype = i64
     lib.orc_int8_round.argtypes = [vp, vp, vp, i32, vp, i32, i32, dbl, dbl,
                                    dbl, vp, vp, vp, dp, dp]
+    lib.orc_adamw_step.restype = None
+    lib.orc_adamw_step.argtypes = [vp, i32, vp, i32, vp, vp, i64, i32, dbl,
+                                   dbl, dbl, dbl, dbl, dbl, i64, vp, vp, vp,
+                                   vp, dp]
     _lib = lib
     return lib
 
@@ -276,3 +280,38 @@ def int8_round(g, v, xs, dtype, parts, mu_t, eta_out, inv_norm, eps=1e-8):
     return {"D": out[0], "C": out[1], "mean_sq_norm": B.value,
             "drift": list(E), "g": g_out, "v": v_out, "x": x_out,
             "nonfinite": int(nf)}
+
+
+# ------------------------------------------------ inner AdamW step (Sec. 2)
+
+def adamw_step(xs, x_dtype, grads, g_dtype, m1s, m2s, lr, beta1, beta2, eps,
+               weight_decay, max_norm, step):
+    """One AdamW step (decoupled weight decay, per-replica gradient-norm
+    clipping) on each replica.  xs / grads: float32 arrays, or bf16 bit
+    patterns (uint16) for dtype BF16; m1s, m2s: float32.  Returns the
+    unrounded float64 results, x' in its storage type and the pre-clipping
+    gradient norms."""
+    M = len(xs)
+    xdt = np.float32 if x_dtype == F32 else np.uint16
+    gdt = np.float32 if g_dtype == F32 else np.uint16
+    xs = [np.ascontiguousarray(a, dtype=xdt) for a in xs]
+    grads = [np.ascontiguousarray(a, dtype=gdt) for a in grads]
+    m1s = [np.ascontiguousarray(a, dtype=np.float32) for a in m1s]
+    m2s = [np.ascontiguousarray(a, dtype=np.float32) for a in m2s]
+    N = xs[0].shape[0]
+    for a in xs + grads + m1s + m2s:
+        assert a.shape == (N,)
+    x_out = [np.empty(N, np.float64) for _ in range(M)]
+    m1_out = [np.empty(N, np.float64) for _ in range(M)]
+    m2_out = [np.empty(N, np.float64) for _ in range(M)]
+    x_store = [np.empty(N, xdt) for _ in range(M)]
+    norms = (ctypes.c_double * M)()
+
+    def arr(lst):
+        return (ctypes.c_void_p * M)(*[_ptr(a) for a in lst])
+    _load().orc_adamw_step(arr(xs), x_dtype, arr(grads), g_dtype, arr(m1s),
+                           arr(m2s), N, M, lr, beta1, beta2, eps,
+                           weight_decay, max_norm, step, arr(x_out),
+                           arr(m1_out), arr(m2_out), arr(x_store), norms)
+    return {"x": x_out, "m1": m1_out, "m2": m2_out, "x_store": x_store,
+            "norms": list(norms)}

@@ -408,3 +408,65 @@ int64_t orc_int8_round(const float *g, const float *v, const void *const *x,
     }
     return nonfinite;
 }
+
+/* ---- inner optimizer: AdamW on every worker (Sec. 2, Eq.
+ * diloco-local-trajectory: each worker takes H local AdamW steps;
+ * Tab. training settings: AdamW coefficients, weight decay, gradient-norm
+ * clipping 1.0, FP32 master parameters and optimizer states) ----
+ *
+ * One step on each of M replicas, written from the definition of AdamW
+ * with decoupled weight decay:
+ *   c      = min(1, max_norm / (||g|| + 1e-6))   (per replica; 1 if max_norm <= 0)
+ *   g~     = c g
+ *   m'     = beta1 m + (1 - beta1) g~
+ *   v'     = beta2 v + (1 - beta2) g~^2
+ *   x'     = x - lr wd x - lr (m' / (1 - beta1^t)) / (sqrt(v' / (1 - beta2^t)) + eps)
+ * with t the 1-based step count.  Readings: the norm is over the whole
+ * replica, the 1e-6 guard and the clipping-factor form are the common
+ * convention (the paper names only the threshold), and the weight decay
+ * applies to every parameter.  x and g may be fp32 or bf16 (widened
+ * exactly); m, v are fp32.  Outputs are unrounded doubles, plus x' in its
+ * storage type (fp32 rounding, or bf16 round-to-nearest-even) when x_store
+ * is given; norms[m] = ||g_m|| before clipping. */
+void orc_adamw_step(const void *const *x, int x_dtype, const void *const *grad,
+                    int g_dtype, const float *const *m1, const float *const *m2,
+                    int64_t N, int M, double lr, double beta1, double beta2,
+                    double eps, double weight_decay, double max_norm,
+                    int64_t step, double *const *x_out, double *const *m1_out,
+                    double *const *m2_out, void *const *x_store, double *norms)
+{
+    double bc1 = 1.0 - pow(beta1, (double)step);
+    double bc2 = 1.0 - pow(beta2, (double)step);
+    for (int m = 0; m < M; ++m) {
+        double ss = 0.0;
+        for (int64_t i = 0; i < N; ++i) {
+            double g = orc_replica(grad[m], g_dtype, i);
+            ss += g * g;
+        }
+        double norm = sqrt(ss);
+        norms[m] = norm;
+        double c = 1.0;
+        if (max_norm > 0.0) {
+            c = max_norm / (norm + 1e-6);
+            if (c > 1.0) c = 1.0;
+        }
+        for (int64_t i = 0; i < N; ++i) {
+            double g = c * orc_replica(grad[m], g_dtype, i);
+            double xv = orc_replica(x[m], x_dtype, i);
+            double mn = beta1 * (double)m1[m][i] + (1.0 - beta1) * g;
+            double vn = beta2 * (double)m2[m][i] + (1.0 - beta2) * g * g;
+            double mhat = mn / bc1;
+            double vhat = vn / bc2;
+            double xn = xv - lr * weight_decay * xv - lr * mhat / (sqrt(vhat) + eps);
+            x_out[m][i] = xn;
+            m1_out[m][i] = mn;
+            m2_out[m][i] = vn;
+            if (x_store && x_store[m]) {
+                if (x_dtype == 0)
+                    ((float *)x_store[m])[i] = (float)xn;
+                else
+                    ((uint16_t *)x_store[m])[i] = orc_double_to_bf16(xn);
+            }
+        }
+    }
+}
