@@ -89,6 +89,7 @@ KERNEL_SOURCES = {
                            "aloco_int8.cu"),
     "int8_fused_kernel": ("aloco_sync_kernel.cuh", "aloco_int8.cuh",
                           "aloco_int8_fused.cu"),
+    "adamw_kernels": ("aloco_sync_kernel.cuh", "aloco_adamw.cu"),
 }
 
 
@@ -526,6 +527,227 @@ def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
             "steps": args.e2e_steps}
 
 
+# ------------------------------------------------------ inner AdamW mode
+
+ADAMW_METRIC = ("inner AdamW steps/s (all M replicas) and achieved HBM GB/s "
+                "(fraction of GB300 roofline) at N params × M replicas")
+ADAMW_UNIT = "steps/s"
+ADAMW_LR, ADAMW_STEP0 = 3e-4, 1200   # a mid-run step of the C4 schedule
+
+
+def adamw_bytes(w) -> int:
+    """Algorithmic HBM bytes of one inner step: per element and replica the
+    parameter (read + write), the gradient (read once) and the two fp32
+    moments (read + write).  Gradients have the replicas' dtype."""
+    r = w.replica_bytes()
+    return w.numel * w.M * (3 * r + 16)
+
+
+def adamw_inputs(w, device, seed=7):
+    """Replicas, gradients (the replicas' dtype; norms about 3, so the
+    C4 threshold of 1.0 clips them) and moments, drawn on `device`."""
+    import torch
+    from paper_2609_36662_gb300 import workloads as W
+    dt = W.replica_dtype(w)
+    gen = torch.Generator(device).manual_seed(seed)
+    sc = 3.0 / max(w.numel, 1) ** 0.5
+
+    def draw(scale, dtype, positive=False):
+        t = torch.empty(w.numel, dtype=torch.float32, device=device)
+        t.normal_(0, 1, generator=gen)
+        if positive:
+            t.abs_()
+        return t.mul_(scale).to(dtype)
+    xs = [draw(0.02, dt) for _ in range(w.M)]
+    gs = [draw(sc, dt) for _ in range(w.M)]
+    m1 = [draw(1e-3 * sc * 30, torch.float32) for _ in range(w.M)]
+    m2 = [draw((sc * 30) ** 2 * 1e-3, torch.float32, True) for _ in range(w.M)]
+    return xs, gs, m1, m2
+
+
+def adamw_oracle_sample(w, xs, gs, m1, m2, elems):
+    """Time the oracle's AdamW step (single thread, as it stands) on the
+    first `elems` elements of every replica.  Returns seconds."""
+    import numpy as np
+    import torch
+    import oracle as O
+    n = min(elems, w.numel)
+
+    def host(t):
+        t = t[:n].cpu()
+        if t.dtype == torch.bfloat16:
+            return t.view(torch.int16).numpy().view(np.uint16)
+        return t.numpy()
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+    hx, hg = [host(t) for t in xs], [host(t) for t in gs]
+    h1, h2 = [host(t) for t in m1], [host(t) for t in m2]
+    t0 = time.perf_counter()
+    O.adamw_step(hx, dt, hg, dt, h1, h2, ADAMW_LR, 0.9, 0.95, 1e-8, 0.1, 1.0,
+                 ADAMW_STEP0)
+    return time.perf_counter() - t0, n
+
+
+def adamw_calibrated(w, xs, gs, m1, m2, target_s):
+    t, n = adamw_oracle_sample(w, xs, gs, m1, m2, min(w.numel, 1 << 18))
+    want = int(target_s / max(t / n, 1e-12))
+    return max(1 << 14, min(w.numel, want))
+
+
+def adamw_config(w):
+    from paper_2609_36662_gb300 import workloads as W
+    return {"workload": w.name, "mode": "adamw", "N": w.numel, "M": w.M,
+            "param_dtype": w.dtype, "grad_dtype": w.dtype,
+            "moment_dtype": "f32",
+            "settings": "C4: lr 3e-4 at step 1200, betas (0.9, 0.95), eps 1e-8, "
+                        "weight decay 0.1, clipping 1.0",
+            "bytes_per_step": adamw_bytes(w),
+            "l2": f"no flush: each step moves {adamw_bytes(w) / 1e9:.1f} GB "
+                  "> 129 MB L2",
+            "parallelism": "replicas only"}
+
+
+def run_adamw_reference(args, w):
+    from paper_2609_36662_gb300 import workloads as W
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    import torch
+    small = W.small(min(w.numel, 1 << 22), w.M, w.dtype)
+    xs, gs, m1, m2 = adamw_inputs(small, "cpu")
+    sample = adamw_calibrated(small, xs, gs, m1, m2, args.ref_step_seconds)
+    times = []
+    for k in range(args.warmup + args.steps):
+        t, n = adamw_oracle_sample(small, xs, gs, m1, m2, sample)
+        if k >= args.warmup:
+            times.append(t)
+    sec = statistics.mean(times) * w.numel / sample
+    value = 1.0 / sec
+    line = {"impl": "reference", "metric": ADAMW_METRIC, "value": value,
+            "unit": ADAMW_UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": sec * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic", "config": adamw_config(w),
+            "cpu_baseline": {"value": value, "unit": ADAMW_UNIT, "cores": 1,
+                             "kind": "oracle",
+                             "sample": f"first {sample} elements of each of "
+                                       f"{w.M} replicas per step, scaled to "
+                                       f"{w.numel}"},
+            "e2e": {"value": value, "unit": ADAMW_UNIT,
+                    "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_adamw(args, w):
+    """Time inner AdamW steps on all replicas (the same gradients every
+    step; parameters and moments evolve)."""
+    import torch
+    from paper_2609_36662_gb300 import aloco as A
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", torch.cuda.current_device())
+    A.load()
+    xs, gs, m1, m2 = adamw_inputs(w, device)
+    stream = torch.cuda.Stream(device)
+    cpu_baseline = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sample = adamw_calibrated(w, xs, gs, m1, m2, args.cpu_seconds)
+        t, n = adamw_oracle_sample(w, xs, gs, m1, m2, sample)
+        cpu_baseline = {"value": (n / w.numel) / t, "unit": ADAMW_UNIT,
+                        "cores": 1, "kind": "oracle",
+                        "sample": f"first {n} of {w.numel} elements of each of "
+                                  f"{w.M} replicas ({t:.1f} s), scaled to a "
+                                  f"full step"}
+    opts = A.default_opts()
+    ev = [(torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True))
+          for _ in range(args.warmup + args.steps)]
+
+    def one_step(k):
+        cfg = A.adamw_cfg(lr=ADAMW_LR, step=ADAMW_STEP0 + k)
+        ev[k][0].record(stream)
+        A.adamw_step(xs, gs, m1, m2, cfg, opts=opts, stream=stream,
+                     want_stats=False)
+        ev[k][1].record(stream)
+
+    for k in range(args.warmup):
+        one_step(k)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(device.index) as clocks:
+        for k in range(args.warmup, args.warmup + args.steps):
+            one_step(k)
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    ms = statistics.mean(ev[k][0].elapsed_time(ev[k][1])
+                         for k in range(args.warmup, args.warmup + args.steps))
+    ms = reduce_max(ms, world, device)
+    st = A.adamw_step(xs, gs, m1, m2, A.adamw_cfg(lr=ADAMW_LR, step=ADAMW_STEP0),
+                      opts=opts, stream=stream)
+    value = job_value(1.0, ms / 1e3, world)
+    peak, peak_kind = hbm_peak()
+    achieved = adamw_bytes(w) / (ms / 1e3) / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        # the step's inputs from pinned host memory (the M gradients), the
+        # step, and the per-replica norms read back
+        hg = [torch.empty_like(g, device="cpu").pin_memory() for g in gs]
+        for a, b in zip(hg, gs):
+            a.copy_(b)
+        times = []
+        for k in range(args.e2e_warmup + args.e2e_steps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            with torch.cuda.stream(stream):
+                for a, b in zip(gs, hg):
+                    a.copy_(b, non_blocking=True)
+            A.adamw_step(xs, gs, m1, m2, A.adamw_cfg(lr=ADAMW_LR,
+                                                     step=ADAMW_STEP0 + k),
+                         opts=opts, stream=stream)
+            e1.record(stream)
+            e1.synchronize()
+            if k >= args.e2e_warmup:
+                times.append(e0.elapsed_time(e1))
+        m_e = reduce_max(statistics.mean(times), world, device)
+        e2e = {"value": job_value(1.0, m_e / 1e3, world), "unit": ADAMW_UNIT,
+               "ms_per_step": m_e,
+               "h2d_bytes_per_step": sum(g.numel() * g.element_size() for g in gs),
+               "d2h_bytes_per_step": 16 * 32, "steps": args.e2e_steps}
+    if rank == 0:
+        line = {
+            "metric": ADAMW_METRIC, "value": value, "unit": ADAMW_UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded replicas, gradients and moments)",
+            "config": adamw_config(w),
+            "elem_per_s": value * w.numel * w.M,
+            "hbm_gbs": achieved,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak,
+                         "peak_source": peak_kind,
+                         "traffic": recorded_traffic(w.name, "adamw_kernels"),
+                         "kernel": "adamw_kernels",
+                         "algorithmic_bytes_per_launch": adamw_bytes(w)},
+            "grad_norms": st["grad_norm"], "clip": st["clip"],
+            "cpu_baseline": cpu_baseline, "e2e": e2e,
+            # two kernels per step: gradient norms, then the update
+            "gpu_launches": 2 * args.steps,
+            "clocks": clocks.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     p.add_argument("--gpus", type=int, default=1)
@@ -546,6 +768,9 @@ def main(argv=None):
     p.add_argument("--comm", choices=["fp32", "int8"], default="fp32",
                    help="int8: the round with INT8-communicated "
                         "pseudo-gradients (App. G.1)")
+    p.add_argument("--mode", choices=["round", "adamw"], default="round",
+                   help="adamw: time the workers' inner AdamW step instead "
+                        "of the outer round")
     p.add_argument("--list", action="store_true")
     args = p.parse_args(argv)
     table = workloads_by_name()
@@ -560,6 +785,9 @@ def main(argv=None):
     if w is None:
         p.error(f"unknown workload {name}; --list shows them, or use "
                 "flat<N>_m<M>_<f32|bf16>")
+    if args.mode == "adamw":
+        return (run_adamw_reference(args, w) if args.impl == "reference"
+                else run_adamw(args, w))
     if args.impl == "reference":
         return run_reference(args, w)
     return run_cuda(args, w)

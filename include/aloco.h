@@ -280,14 +280,77 @@ int aloco_int8_decode(const int8_t *codes, const float *scales, size_t N,
  * and decoded once, and that aggregate drives the corrected Nesterov step and
  * the replica reset.  D_t and the drift energies use the pre-quantisation
  * pseudo-gradients, C_t and ||Dbar||^2 the decoded aggregate.  Arguments as
- * aloco_sync_ex plus the parts; M <= 16; opts->pass and blocks_per_sm do not
- * apply (one kernel runs it). */
+ * aloco_sync_ex plus the parts; M <= 16; opts->pass selects the form
+ * (AUTO, INT8_SPLIT or INT8_FUSED; see aloco_pass) and blocks_per_sm does
+ * not apply. */
 int aloco_sync_int8(float *global, float *momentum, void *const *locals,
                     size_t N, int M, aloco_dtype dtype, int64_t H_sel,
                     int64_t H_base, int64_t step,
                     const aloco_schedule_t *schedule, double outer_lr,
                     double outer_beta, const int64_t *part_sizes, int n_parts,
                     const aloco_opts_t *opts, aloco_stats_t *stats_out);
+
+/* ------------------------------------------------------------------------
+ * Inner optimizer (Sec. 2, Eq. diloco-local-trajectory: every worker takes
+ * H local AdamW steps between synchronisations; Tab. training settings:
+ * AdamW coefficients (0.9, 0.95) for C4 and (0.9, 0.999) for SFT, weight
+ * decay 0.1 / 0, gradient-norm clipping 1.0, FP32 master parameters and
+ * optimizer states).  The paper's runs compute the gradients from data; this
+ * library takes them as inputs, so a caller can drive whole intervals on one
+ * GPU with synthetic gradients.
+ *
+ * One step on each of the M replicas:
+ *   c_m = min(1, max_grad_norm / (||g_m|| + 1e-6))   (1 if max_grad_norm <= 0)
+ *   m'  = beta1 m + (1 - beta1) c_m g
+ *   v'  = beta2 v + (1 - beta2) (c_m g)^2
+ *   x'  = x - lr weight_decay x
+ *           - lr (m' / (1 - beta1^step)) / (sqrt(v' / (1 - beta2^step)) + eps)
+ * in fp32 arithmetic per element; ||g_m|| is summed in fp64 over the whole
+ * replica in a fixed order.
+ * ---------------------------------------------------------------------- */
+
+typedef struct aloco_adamw_cfg {
+    double lr;             /* this step's inner learning rate eta_{t,h} > 0  */
+    double beta1;          /* first-moment coefficient, in [0, 1)            */
+    double beta2;          /* second-moment coefficient, in [0, 1)           */
+    double eps;            /* denominator guard, > 0                         */
+    double weight_decay;   /* decoupled decay coefficient, >= 0              */
+    double max_grad_norm;  /* per-replica clipping threshold; <= 0: none     */
+    int64_t step;          /* 1-based index of this step (bias correction)   */
+} aloco_adamw_cfg_t;
+
+/* Per-replica results of one step. */
+typedef struct aloco_adamw_stats {
+    double grad_norm[ALOCO_MAX_WORKERS];  /* ||g_m|| before clipping         */
+    double clip[ALOCO_MAX_WORKERS];       /* c_m applied                     */
+    int32_t M;
+    int32_t grid;                         /* CUDA blocks of the update pass  */
+    float kernel_ms;                      /* both passes, or -1              */
+    int32_t reserved;
+} aloco_adamw_stats_t;
+
+/* The C4 pre-training settings: lr 4e-4, (0.9, 0.95), eps 1e-8, weight
+ * decay 0.1, clipping at 1.0, step 1. */
+void aloco_adamw_default_cfg(aloco_adamw_cfg_t *cfg);
+
+/* One AdamW step on M <= ALOCO_MAX_WORKERS replicas, in place.
+ *   params[m]     x_m, N elements of param_dtype (fp32 or bf16; bf16 results
+ *                 are rounded to nearest even), updated;
+ *   grads[m]      g_m, N elements of grad_dtype, read only;
+ *   exp_avg[m], exp_avg_sq[m]   m and v, fp32, updated.
+ * Host arrays of M device pointers to caller-owned device memory of the
+ * current device; no two updated buffers may overlap.  opts (NULL =
+ * defaults) supplies the stream, kernel timing and blocks_per_sm; the
+ * correction and pass fields do not apply.  With stats_out == NULL the call
+ * only enqueues its two kernels; otherwise it waits for them and fills
+ * *stats_out.  Returns ALOCO_OK, ALOCO_ERR_ARG / ALOCO_ERR_ALIAS before any
+ * device work, or ALOCO_ERR_CUDA.  Calls on one device share its scratch:
+ * steps that overlap on the GPU (different streams, no ordering) race. */
+int aloco_adamw_step(void *const *params, const void *const *grads,
+                     float *const *exp_avg, float *const *exp_avg_sq, size_t N,
+                     int M, aloco_dtype param_dtype, aloco_dtype grad_dtype,
+                     const aloco_adamw_cfg_t *cfg, const aloco_opts_t *opts,
+                     aloco_adamw_stats_t *stats_out);
 
 /* ------------------------------------------------------------------------
  * Interval controller (Sec. 3.1; App. A).  Host-only and scalar: after each

@@ -33,7 +33,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
 EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
            "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc",
            "aloco_sync_int8", "aloco_int8_num_blocks", "aloco_int8_encode",
-           "aloco_int8_decode",
+           "aloco_int8_decode", "aloco_adamw_default_cfg", "aloco_adamw_step",
            "aloco_ctrl_default_cfg", "aloco_ctrl_init", "aloco_select_interval",
            "aloco_ctrl_state_bytes", "aloco_ctrl_save", "aloco_ctrl_load",
            "aloco_last_error", "aloco_shutdown", "aloco_version")
@@ -65,6 +65,25 @@ class Opts(ctypes.Structure):
                 ("blocks_per_sm", ctypes.c_int32),
                 ("stream", ctypes.c_void_p), ("pass_", ctypes.c_int32),
                 ("reserved", ctypes.c_int32)]
+
+
+class AdamwCfg(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_double), ("beta1", ctypes.c_double),
+                ("beta2", ctypes.c_double), ("eps", ctypes.c_double),
+                ("weight_decay", ctypes.c_double),
+                ("max_grad_norm", ctypes.c_double), ("step", ctypes.c_int64)]
+
+
+class AdamwStats(ctypes.Structure):
+    _fields_ = [("grad_norm", ctypes.c_double * MAX_WORKERS),
+                ("clip", ctypes.c_double * MAX_WORKERS),
+                ("M", ctypes.c_int32), ("grid", ctypes.c_int32),
+                ("kernel_ms", ctypes.c_float), ("reserved", ctypes.c_int32)]
+
+    def as_dict(self):
+        return {"grad_norm": list(self.grad_norm[:self.M]),
+                "clip": list(self.clip[:self.M]), "M": self.M,
+                "grid": self.grid, "kernel_ms": self.kernel_ms}
 
 
 class Correction(ctypes.Structure):
@@ -183,6 +202,12 @@ def load():
     P = ctypes.POINTER
     lib.aloco_sync_int8.argtypes = sync_args + [vp, i32, P(Opts), P(Stats)]
     lib.aloco_sync_int8.restype = i32
+    lib.aloco_adamw_default_cfg.argtypes = [P(AdamwCfg)]
+    lib.aloco_adamw_default_cfg.restype = None
+    lib.aloco_adamw_step.argtypes = [vp, vp, vp, vp, ctypes.c_size_t, i32,
+                                     i32, i32, P(AdamwCfg), P(Opts),
+                                     P(AdamwStats)]
+    lib.aloco_adamw_step.restype = i32
     lib.aloco_int8_num_blocks.argtypes = [vp, i32]
     lib.aloco_int8_num_blocks.restype = i64
     lib.aloco_int8_encode.argtypes = [vp, ctypes.c_size_t, vp, i32, vp, vp, vp,
@@ -450,4 +475,53 @@ def sync_int8(global_, momentum, locals_, *, parts=None, H_sel: int,
                                     ctypes.byref(st))
     if raise_on_error and rc not in (OK, ERR_NONFINITE):
         raise AlocoError(rc, last_error())
+    return st.as_dict() | {"status": rc}
+
+
+# ----------------------------------------------------- inner AdamW (Sec. 2)
+
+def adamw_cfg(**kw) -> AdamwCfg:
+    """The library's default AdamW settings (C4 pre-training) with the given
+    fields replaced."""
+    c = AdamwCfg()
+    load().aloco_adamw_default_cfg(ctypes.byref(c))
+    for k, v in kw.items():
+        if not hasattr(c, k):
+            raise TypeError(f"unknown AdamW setting {k!r}")
+        setattr(c, k, v)
+    return c
+
+
+def adamw_step(params, grads, exp_avg, exp_avg_sq, cfg: AdamwCfg,
+               opts: Optional[Opts] = None, stream=None, want_stats=True,
+               raise_on_error=True):
+    """One AdamW step on every replica, in place (lists of torch CUDA tensors
+    of one device: params and grads fp32 or bf16, moments fp32).  Returns the
+    per-replica gradient norms and clipping factors (want_stats), else None
+    without waiting for the GPU."""
+    import torch
+    M = len(params)
+    if not (len(grads) == len(exp_avg) == len(exp_avg_sq) == M):
+        raise ValueError("params, grads and moments need one tensor per replica")
+    N = params[0].numel()
+    pdt = F32 if params[0].dtype == torch.float32 else BF16
+    gdt = F32 if grads[0].dtype == torch.float32 else BF16
+    if opts is None:
+        opts = default_opts()
+    s = stream if stream is not None else torch.cuda.current_stream(
+        params[0].device)
+    opts.stream = s.cuda_stream
+
+    def arr(ts):
+        return (ctypes.c_void_p * M)(*[t.data_ptr() for t in ts])
+    st = AdamwStats() if want_stats else None
+    with torch.cuda.device(params[0].device):
+        rc = load().aloco_adamw_step(arr(params), arr(grads), arr(exp_avg),
+                                     arr(exp_avg_sq), N, M, pdt, gdt,
+                                     ctypes.byref(cfg), ctypes.byref(opts),
+                                     ctypes.byref(st) if st is not None else None)
+    if raise_on_error and rc != OK:
+        raise AlocoError(rc, last_error())
+    if st is None:
+        return rc if not raise_on_error else None
     return st.as_dict() | {"status": rc}

@@ -5,6 +5,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -174,6 +175,8 @@ struct Workspace {
     unsigned long long *nf_total = nullptr;
     unsigned int *error = nullptr;
     unsigned int *ticket = nullptr;
+    double *adam = nullptr;               // AdamW: [max_grid] partials, then
+                                          // [2 * MAX_WORKERS] norms and factors
     char *i8 = nullptr;                   // INT8 round scratch (grown on demand)
     size_t i8_cap = 0;
     double *host = nullptr;               // pinned readback of totals + nf
@@ -181,6 +184,8 @@ struct Workspace {
 };
 
 constexpr int kTotals = aloco::kTotalsSlots;
+// pinned read-back slots: the round's totals, or AdamW's norms and factors
+constexpr int kHostSlots = kTotals > 2 * ALOCO_MAX_WORKERS ? kTotals : 2 * ALOCO_MAX_WORKERS;
 
 std::mutex g_registry_mu;
 std::vector<std::unique_ptr<Workspace>> g_registry;
@@ -204,9 +209,10 @@ int ensure_ready(Workspace *ws, int device) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
     ws->max_grid = ws->sm_count * (max_threads / aloco::kBlock);
     const size_t n_part = (size_t)ws->max_grid * (ALOCO_MAX_WORKERS + 1);
+    const size_t n_adam = (size_t)ws->max_grid + 2 * ALOCO_MAX_WORKERS;
     const size_t bytes = n_part * sizeof(double) +
                          (size_t)ws->max_grid * sizeof(unsigned long long) +
-                         kTotals * sizeof(double) + 256;
+                         kTotals * sizeof(double) + n_adam * sizeof(double) + 256;
     e = cudaMalloc((void **)&ws->dev, bytes);
     if (e != cudaSuccess) {
         cudaGetLastError();
@@ -222,9 +228,11 @@ int ensure_ready(Workspace *ws, int device) {
     ws->nf_total = (unsigned long long *)(ws->totals + aloco::kNfSlot);
     ws->error = (unsigned int *)(ws->totals + aloco::kErrorSlot);
     p += kTotals * sizeof(double);
+    ws->adam = (double *)p;
+    p += n_adam * sizeof(double);
     ws->ticket = (unsigned int *)p;
     e = cudaMemset(ws->dev, 0, bytes);
-    if (e == cudaSuccess) e = cudaMallocHost((void **)&ws->host, kTotals * sizeof(double));
+    if (e == cudaSuccess) e = cudaMallocHost((void **)&ws->host, kHostSlots * sizeof(double));
     if (e == cudaSuccess) e = cudaEventCreate(&ws->ev0);
     if (e == cudaSuccess) e = cudaEventCreate(&ws->ev1);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -732,6 +740,186 @@ int aloco_int8_decode(const int8_t *codes, const float *scales, size_t N,
     cudaError_t e = aloco::launch_int8_decode(codes, scales, out, vec, P, sms,
                                               (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "int8 decode launch");
+    t_err.clear();
+    return ALOCO_OK;
+}
+
+void aloco_adamw_default_cfg(aloco_adamw_cfg_t *cfg) {
+    if (!cfg) return;
+    std::memset(cfg, 0, sizeof *cfg);
+    cfg->lr = 4e-4;
+    cfg->beta1 = 0.9;
+    cfg->beta2 = 0.95;
+    cfg->eps = 1e-8;
+    cfg->weight_decay = 0.1;
+    cfg->max_grad_norm = 1.0;
+    cfg->step = 1;
+}
+
+int aloco_adamw_step(void *const *params, const void *const *grads,
+                     float *const *exp_avg, float *const *exp_avg_sq, size_t N,
+                     int M, aloco_dtype param_dtype, aloco_dtype grad_dtype,
+                     const aloco_adamw_cfg_t *cfg, const aloco_opts_t *opts,
+                     aloco_adamw_stats_t *stats_out) {
+    aloco_opts_t o;
+    if (opts) o = *opts; else fill_default_opts(&o);
+    if (!cfg) return fail(ALOCO_ERR_ARG, "NULL cfg");
+    if (M < 1 || M > ALOCO_MAX_WORKERS)
+        return fail(ALOCO_ERR_ARG, "M = %d outside [1, %d]", M, ALOCO_MAX_WORKERS);
+    if ((param_dtype != ALOCO_F32 && param_dtype != ALOCO_BF16) ||
+        (grad_dtype != ALOCO_F32 && grad_dtype != ALOCO_BF16))
+        return fail(ALOCO_ERR_ARG, "unknown dtype (params %d, grads %d)",
+                    (int)param_dtype, (int)grad_dtype);
+    const aloco_adamw_cfg_t &c = *cfg;
+    if (!(std::isfinite(c.lr) && c.lr >= 0.0))
+        return fail(ALOCO_ERR_ARG, "lr = %g must be finite and >= 0", c.lr);
+    if (!(c.beta1 >= 0.0 && c.beta1 < 1.0) || !(c.beta2 >= 0.0 && c.beta2 < 1.0))
+        return fail(ALOCO_ERR_ARG, "betas (%g, %g) must lie in [0, 1)", c.beta1, c.beta2);
+    if (!(std::isfinite(c.eps) && c.eps > 0.0))
+        return fail(ALOCO_ERR_ARG, "eps = %g must be finite and > 0", c.eps);
+    if (!(std::isfinite(c.weight_decay) && c.weight_decay >= 0.0))
+        return fail(ALOCO_ERR_ARG, "weight_decay = %g must be finite and >= 0",
+                    c.weight_decay);
+    if (!std::isfinite(c.max_grad_norm))
+        return fail(ALOCO_ERR_ARG, "max_grad_norm must be finite");
+    if (c.step < 1) return fail(ALOCO_ERR_ARG, "step = %lld must be >= 1", (long long)c.step);
+    if (o.blocks_per_sm < 0)
+        return fail(ALOCO_ERR_ARG, "blocks_per_sm = %d must be >= 0", o.blocks_per_sm);
+    if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
+    if (N > 0 && (!params || !grads || !exp_avg || !exp_avg_sq))
+        return fail(ALOCO_ERR_ARG, "NULL pointer array");
+    for (int m = 0; N > 0 && m < M; ++m)
+        if (!params[m] || !grads[m] || !exp_avg[m] || !exp_avg_sq[m])
+            return fail(ALOCO_ERR_ARG, "NULL buffer for replica %d", m);
+
+    aloco_adamw_stats_t local;
+    aloco_adamw_stats_t *st = stats_out ? stats_out : &local;
+    std::memset(st, 0, sizeof *st);
+    st->M = M;
+    st->kernel_ms = -1.f;
+    for (int m = 0; m < M; ++m) st->clip[m] = 1.0;
+    if (N == 0) {
+        t_err.clear();
+        return ALOCO_OK;
+    }
+
+    const size_t psz = param_dtype == ALOCO_F32 ? 4 : 2;
+    const size_t gsz = grad_dtype == ALOCO_F32 ? 4 : 2;
+    // Updated buffers may overlap nothing; gradients may be shared by
+    // replicas (read only) but may not overlap an updated buffer.
+    {
+        std::vector<std::pair<uintptr_t, size_t>> upd, rd;
+        for (int m = 0; m < M; ++m) {
+            upd.push_back({(uintptr_t)params[m], N * psz});
+            upd.push_back({(uintptr_t)exp_avg[m], N * 4});
+            upd.push_back({(uintptr_t)exp_avg_sq[m], N * 4});
+            rd.push_back({(uintptr_t)grads[m], N * gsz});
+        }
+        auto hit = [](const std::pair<uintptr_t, size_t> &a,
+                      const std::pair<uintptr_t, size_t> &b) {
+            return a.first < b.first + b.second && b.first < a.first + a.second;
+        };
+        for (size_t i = 0; i < upd.size(); ++i) {
+            for (size_t j = i + 1; j < upd.size(); ++j)
+                if (hit(upd[i], upd[j]))
+                    return fail(ALOCO_ERR_ALIAS, "updated buffers %zu and %zu overlap", i, j);
+            for (size_t j = 0; j < rd.size(); ++j)
+                if (hit(upd[i], rd[j]))
+                    return fail(ALOCO_ERR_ALIAS, "grads[%zu] overlaps an updated buffer", j);
+        }
+    }
+    uintptr_t align_or = 0;
+    for (int m = 0; m < M; ++m) {
+        if (((uintptr_t)params[m] & (psz - 1)) || ((uintptr_t)grads[m] & (gsz - 1)) ||
+            ((uintptr_t)exp_avg[m] & 3) || ((uintptr_t)exp_avg_sq[m] & 3))
+            return fail(ALOCO_ERR_ARG, "replica %d: buffer not aligned to its element", m);
+        align_or |= (uintptr_t)params[m] | (uintptr_t)grads[m] |
+                    (uintptr_t)exp_avg[m] | (uintptr_t)exp_avg_sq[m];
+    }
+
+    int device = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    Workspace *ws = workspace_for(device);
+    std::lock_guard<std::mutex> lk(ws->mu);
+    int rc = ensure_ready(ws, device);
+    if (rc != ALOCO_OK) return rc;
+    for (int m = 0; m < M; ++m) {
+        char name[40];
+        snprintf(name, sizeof name, "params[%d]", m);
+        if ((rc = check_buffer(params[m], N * psz, device, name)) != ALOCO_OK) return rc;
+        snprintf(name, sizeof name, "grads[%d]", m);
+        if ((rc = check_buffer(grads[m], N * gsz, device, name)) != ALOCO_OK) return rc;
+        snprintf(name, sizeof name, "exp_avg[%d]", m);
+        if ((rc = check_buffer(exp_avg[m], N * 4, device, name)) != ALOCO_OK) return rc;
+        snprintf(name, sizeof name, "exp_avg_sq[%d]", m);
+        if ((rc = check_buffer(exp_avg_sq[m], N * 4, device, name)) != ALOCO_OK) return rc;
+    }
+
+    aloco::AdamArgs a;
+    std::memset(&a, 0, sizeof a);
+    for (int m = 0; m < M; ++m) {
+        a.x[m] = params[m];
+        a.g[m] = grads[m];
+        a.m1[m] = exp_avg[m];
+        a.m2[m] = exp_avg_sq[m];
+    }
+    a.n = (int64_t)N;
+    a.nunit = (align_or & 15) == 0 ? (int64_t)(N / 4) : 0;
+    a.M = M;
+    const double bc1 = 1.0 - std::pow(c.beta1, (double)c.step);
+    const double bc2 = 1.0 - std::pow(c.beta2, (double)c.step);
+    a.beta1 = (float)c.beta1;
+    a.omb1 = (float)(1.0 - c.beta1);
+    a.beta2 = (float)c.beta2;
+    a.omb2 = (float)(1.0 - c.beta2);
+    a.decay = (float)(1.0 - c.lr * c.weight_decay);
+    a.neg_step = (float)(-c.lr / bc1);
+    a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
+    a.eps = (float)c.eps;
+    a.max_norm = c.max_grad_norm;
+    a.partials = ws->adam;
+    a.out = ws->adam + ws->max_grid;
+
+    // norm pass: up to the workspace's max_grid blocks over all workers;
+    // update pass: SMs x blocks_per_sm blocks (default 4) over all workers
+    const int64_t work = a.nunit > 0 ? a.nunit : a.n;
+    const int64_t per_thread = (int64_t)aloco::kBlock;
+    int64_t g1 = ws->max_grid / M;
+    g1 = std::min<int64_t>(g1, (work + per_thread - 1) / per_thread);
+    a.g1 = (int)std::max<int64_t>(g1, 1);
+    const int bps = o.blocks_per_sm > 0 ? o.blocks_per_sm : 4;
+    int64_t g2 = ((int64_t)ws->sm_count * bps + M - 1) / M;
+    g2 = std::min<int64_t>(g2, (work + 2 * per_thread - 1) / (2 * per_thread));
+    g2 = std::max<int64_t>(g2, 1);
+    if (g2 > 65535) g2 = 65535;
+
+    cudaStream_t stream = (cudaStream_t)o.stream;
+    const bool timed = o.time_kernel && stats_out;
+    if (timed && (e = cudaEventRecord(ws->ev0, stream)) != cudaSuccess)
+        return cuda_fail(e, "cudaEventRecord");
+    e = aloco::launch_adamw(a, param_dtype, grad_dtype, (int)g2, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "AdamW launch");
+    if (timed && (e = cudaEventRecord(ws->ev1, stream)) != cudaSuccess)
+        return cuda_fail(e, "cudaEventRecord");
+    st->grid = (int)(g2 * M);
+    if (stats_out) {
+        e = cudaMemcpyAsync(ws->host, a.out, 2 * ALOCO_MAX_WORKERS * sizeof(double),
+                            cudaMemcpyDeviceToHost, stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+        if (e != cudaSuccess) return cuda_fail(e, "AdamW step");
+        for (int m = 0; m < M; ++m) {
+            st->grad_norm[m] = ws->host[m];
+            st->clip[m] = ws->host[ALOCO_MAX_WORKERS + m];
+        }
+        if (timed) {
+            float ms = -1.f;
+            if (cudaEventElapsedTime(&ms, ws->ev0, ws->ev1) == cudaSuccess)
+                st->kernel_ms = ms;
+            else
+                cudaGetLastError();
+        }
+    }
     t_err.clear();
     return ALOCO_OK;
 }

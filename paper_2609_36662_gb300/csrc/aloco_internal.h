@@ -114,6 +114,32 @@ cudaError_t launch_int8_decode(const int8_t *codes, const float *scales,
                                float *out, bool vec_ok, const Int8Parts &P,
                                int sm_count, cudaStream_t stream);
 
+// One AdamW step on M replicas (aloco_adamw.cu), passed by value.
+struct AdamArgs {
+    void *x[ALOCO_MAX_WORKERS];         // parameters [n] (fp32 or bf16)
+    const void *g[ALOCO_MAX_WORKERS];   // gradients [n] (fp32 or bf16)
+    float *m1[ALOCO_MAX_WORKERS];       // first moments [n]
+    float *m2[ALOCO_MAX_WORKERS];       // second moments [n]
+    int64_t n;                          // elements per replica
+    int64_t nunit;                      // 4-element units of the vector loop
+                                        // (0 when a buffer is not 16 B aligned)
+    int M;
+    int g1;                             // norm-pass blocks per worker
+    float beta1, omb1;                  // beta1, 1 - beta1
+    float beta2, omb2;                  // beta2, 1 - beta2
+    float decay;                        // 1 - lr * weight_decay
+    float neg_step;                     // -lr / (1 - beta1^step)
+    float inv_sqrt_bc2;                 // 1 / sqrt(1 - beta2^step)
+    float eps;
+    double max_norm;                    // clipping threshold; <= 0: none
+    double *partials;                   // [M][g1] sums of g^2 (device)
+    double *out;                        // [2][ALOCO_MAX_WORKERS]: norms, factors
+};
+
+// Enqueue the norm pass (grid g1 x M) and the update pass (grid g2 x M).
+cudaError_t launch_adamw(const AdamArgs &a, aloco_dtype param_dtype,
+                         aloco_dtype grad_dtype, int g2, cudaStream_t stream);
+
 // Host helpers shared by the entry points (aloco_host.cpp).
 int report_error(int code, const char *msg);
 int check_buffer(const void *p, size_t bytes, int device, const char *name);

@@ -64,6 +64,9 @@ int main(void) {
          offsetof(aloco_stats_t, corr), offsetof(aloco_stats_t, nonfinite),
          offsetof(aloco_stats_t, kernel_ms), offsetof(aloco_schedule_t, peak_lr),
          offsetof(aloco_schedule_t, total_steps));
+  printf("%zu %zu %zu %zu %zu\n", sizeof(aloco_adamw_cfg_t),
+         sizeof(aloco_adamw_stats_t), offsetof(aloco_adamw_cfg_t, step),
+         offsetof(aloco_adamw_stats_t, clip), offsetof(aloco_adamw_stats_t, kernel_ms));
   return 0;
 }
 ''')
@@ -80,6 +83,10 @@ int main(void) {
                     A.CtrlState.hist_C.offset, A.CtrlState.referenced.offset]
     assert sizes == [ctypes.sizeof(A.Schedule), ctypes.sizeof(A.Opts),
                      ctypes.sizeof(A.Correction), ctypes.sizeof(A.Stats)]
+    adam = list(map(int, lines[3].split()))
+    assert adam == [ctypes.sizeof(A.AdamwCfg), ctypes.sizeof(A.AdamwStats),
+                    A.AdamwCfg.step.offset, A.AdamwStats.clip.offset,
+                    A.AdamwStats.kernel_ms.offset]
     assert offs == [A.Opts.pass_.offset, A.Opts.stream.offset,
                     A.Stats.corr.offset,
                     A.Stats.nonfinite.offset, A.Stats.kernel_ms.offset,
@@ -274,3 +281,46 @@ def test_int8_block_count_gives_the_papers_payload(lib):
     for bad in ([0], [5, -1]):
         with pytest.raises(A.AlocoError):
             A.int8_num_blocks(bad)
+
+
+def test_adamw_defaults_and_argument_errors(lib):
+    """Default settings are the C4 pre-training recipe (Tab. training
+    settings); bad settings, NULLs and overlapping buffers are rejected
+    before any device work."""
+    import ctypes
+    c = A.adamw_cfg()
+    assert (c.lr, c.beta1, c.beta2, c.eps, c.weight_decay, c.max_grad_norm,
+            c.step) == (4e-4, 0.9, 0.95, 1e-8, 0.1, 1.0, 1)
+    base = 1 << 40
+    MB = 1 << 20
+
+    def call(cfg=None, N=1000, M=2, pdt=A.F32, gdt=A.F32, ptrs=None):
+        cfg = cfg or A.adamw_cfg()
+        p = ptrs or {k: [base + (4 * m + i) * MB for m in range(M)]
+                     for i, k in enumerate(("x", "g", "m1", "m2"))}
+        arr = lambda v: (ctypes.c_void_p * M)(*v)
+        return lib.aloco_adamw_step(arr(p["x"]), arr(p["g"]), arr(p["m1"]),
+                                    arr(p["m2"]), N, M, pdt, gdt,
+                                    ctypes.byref(cfg), None, None)
+    for kw in (dict(lr=-1.0), dict(beta1=1.0), dict(beta2=-0.1), dict(eps=0.0),
+               dict(weight_decay=-0.1), dict(max_grad_norm=float("nan")),
+               dict(step=0)):
+        assert call(A.adamw_cfg(**kw)) == A.ERR_ARG, kw
+    assert call(M=0) == A.ERR_ARG
+    assert call(M=33) == A.ERR_ARG
+    assert call(pdt=7) == A.ERR_ARG
+    # a moment buffer overlapping a parameter buffer
+    p = {"x": [base, base + MB], "g": [base + 2 * MB, base + 3 * MB],
+         "m1": [base + 4 * MB, base + 100], "m2": [base + 6 * MB, base + 7 * MB]}
+    assert call(ptrs=p) == A.ERR_ALIAS
+    # a gradient overlapping an updated buffer
+    p = {"x": [base, base + MB], "g": [base + 8, base + 3 * MB],
+         "m1": [base + 4 * MB, base + 5 * MB], "m2": [base + 6 * MB, base + 7 * MB]}
+    assert call(ptrs=p) == A.ERR_ALIAS
+    # one gradient shared by both replicas passes the argument checks
+    p = {"x": [base, base + MB], "g": [base + 2 * MB] * 2,
+         "m1": [base + 4 * MB, base + 5 * MB], "m2": [base + 6 * MB, base + 7 * MB]}
+    assert call(ptrs=p) in (A.ERR_CUDA, A.ERR_ARG)
+    assert "overlap" not in A.last_error()
+    # N = 0 needs no device
+    assert call(N=0) == A.OK
