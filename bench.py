@@ -468,6 +468,11 @@ def run_cuda(args, w):
 
 def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
             int8_parts=None):
+    """The metric end to end with the state in pinned host memory.  The
+    plain round goes through aloco_sync_host (the library streams theta, v
+    and the endpoints to the GPU and theta', v' back in overlapped chunks);
+    the INT8 round copies the inputs in, calls aloco_sync_int8 and copies
+    theta', v' out."""
     import torch
     from paper_2609_36662_gb300 import aloco as A
     from paper_2609_36662_gb300 import workloads as W
@@ -486,37 +491,39 @@ def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
     hv = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
     hx = [torch.empty(w.numel, dtype=W.replica_dtype(w), pin_memory=True)
           for _ in range(w.M)]
-    og = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
-    ov = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
     W.fill_replicas(w, g, xs, 0)
     hg.copy_(g)
     hv.copy_(v)
     for a, b in zip(hx, xs):
         a.copy_(b)
+    og = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
+    ov = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
     ms = []
     n_total = args.e2e_warmup + args.e2e_steps
     for k in range(n_total):
         step, hsel = rounds[k % len(rounds)]
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
-        with torch.cuda.stream(stream):
-            e0.record(stream)
-            g.copy_(hg, non_blocking=True)
-            v.copy_(hv, non_blocking=True)
-            for a, b in zip(xs, hx):
-                a.copy_(b, non_blocking=True)
-            if int8_parts is not None:
-                A.sync_int8(g, v, xs, parts=int8_parts, H_sel=hsel,
-                            H_base=w.H_base, step=step, schedule=sched,
-                            outer_lr=w.outer_lr, outer_beta=w.outer_beta,
-                            stream=stream)
-            else:
-                A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step,
-                       schedule=sched, outer_lr=w.outer_lr,
-                       outer_beta=w.outer_beta, stream=stream)
-            og.copy_(g, non_blocking=True)
-            ov.copy_(v, non_blocking=True)
-            e1.record(stream)
+        e0.record(stream)
+        if int8_parts is None:
+            # theta' and v' come back into hg, hv (the next round's inputs)
+            A.sync_host(hg, hv, hx, H_sel=hsel, H_base=w.H_base, step=step,
+                        schedule=sched, outer_lr=w.outer_lr,
+                        outer_beta=w.outer_beta, stream=stream)
+        else:
+            with torch.cuda.stream(stream):
+                g.copy_(hg, non_blocking=True)
+                v.copy_(hv, non_blocking=True)
+                for a, b in zip(xs, hx):
+                    a.copy_(b, non_blocking=True)
+            A.sync_int8(g, v, xs, parts=int8_parts, H_sel=hsel,
+                        H_base=w.H_base, step=step, schedule=sched,
+                        outer_lr=w.outer_lr, outer_beta=w.outer_beta,
+                        stream=stream)
+            with torch.cuda.stream(stream):
+                og.copy_(g, non_blocking=True)
+                ov.copy_(v, non_blocking=True)
+        e1.record(stream)
         e1.synchronize()
         if k >= args.e2e_warmup:
             ms.append(e0.elapsed_time(e1))
@@ -524,7 +531,9 @@ def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
     return {"value": job_value(1.0, m / 1e3, world), "unit": UNIT,
             "ms_per_step": m, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h + 8 * (w.M + 2),
-            "steps": args.e2e_steps}
+            "steps": args.e2e_steps,
+            "api": "aloco_sync_host" if int8_parts is None else
+                   "copies + aloco_sync_int8"}
 
 
 # ------------------------------------------------------ inner AdamW mode

@@ -244,6 +244,33 @@ int aloco_sync_ex(float *global, float *momentum, void *const *locals,
                   double outer_beta, const aloco_opts_t *opts,
                   aloco_stats_t *stats_out);
 
+/* One outer round (as aloco_sync_ex, Algorithm 1) on state that lives in
+ * host memory: theta, v and the M replicas are page-locked host arrays
+ * (cudaMallocHost, or registered with cudaHostRegister); any other memory
+ * is ALOCO_ERR_ARG.  The library streams them through cached device
+ * staging in chunks of chunk_elems elements (0 = 2^24; rounded up to a
+ * multiple of 8), overlapping the host-to-device copy of one chunk, the
+ * fused kernel on another and the device-to-host copy of theta' and v' of a
+ * third, on two internal copy streams and opts->stream.
+ *   global, momentum  in: theta, v; out: theta', v' (fp32, N each);
+ *   locals            in only: the replicas' endpoints.  The host replicas
+ *                     are NOT reset; the reset replicas equal theta', which
+ *                     the caller hands to its workers.
+ * Per-element results are bit-identical to aloco_sync_ex on the same
+ * inputs; the statistics differ only in the grouping of their partial sums
+ * (fp32 per thread, then fp64), so in their last few fp32 bits.  The register
+ * pass runs (opts->pass AUTO or REGISTERS; BULK_COPY is ALOCO_ERR_ARG).
+ * The call returns when theta', v' and the statistics are in place.  The
+ * device staging (3 chunks of (8 + M * element size) bytes each) is
+ * allocated on first use, kept until aloco_shutdown, and shared by the
+ * device's calls, which therefore must not overlap. */
+int aloco_sync_host(float *global, float *momentum, const void *const *locals,
+                    size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                    int64_t H_base, int64_t step,
+                    const aloco_schedule_t *schedule, double outer_lr,
+                    double outer_beta, size_t chunk_elems,
+                    const aloco_opts_t *opts, aloco_stats_t *stats_out);
+
 /* ------------------------------------------------------------------------
  * INT8 pseudo-gradient communication (App. G.1).
  *

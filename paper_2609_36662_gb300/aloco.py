@@ -31,7 +31,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
 
 # Names declared in include/aloco.h (checked by the ABI test).
 EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
-           "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc",
+           "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc", "aloco_sync_host",
            "aloco_sync_int8", "aloco_int8_num_blocks", "aloco_int8_encode",
            "aloco_int8_decode", "aloco_adamw_default_cfg", "aloco_adamw_step",
            "aloco_ctrl_default_cfg", "aloco_ctrl_init", "aloco_select_interval",
@@ -208,6 +208,8 @@ def load():
                                      i32, i32, P(AdamwCfg), P(Opts),
                                      P(AdamwStats)]
     lib.aloco_adamw_step.restype = i32
+    lib.aloco_sync_host.argtypes = sync_args + [ctypes.c_size_t, P(Opts), P(Stats)]
+    lib.aloco_sync_host.restype = i32
     lib.aloco_int8_num_blocks.argtypes = [vp, i32]
     lib.aloco_int8_num_blocks.restype = i64
     lib.aloco_int8_encode.argtypes = [vp, ctypes.c_size_t, vp, i32, vp, vp, vp,
@@ -446,6 +448,31 @@ def int8_decode(codes, scales, parts=None, stream=None):
     if rc != OK:
         raise AlocoError(rc, last_error())
     return out
+
+
+def sync_host(global_, momentum, locals_, *, H_sel: int, H_base: int,
+              step: int, schedule: Schedule, outer_lr: float,
+              outer_beta: float, chunk_elems: int = 0,
+              opts: Optional[Opts] = None, stream=None, raise_on_error=True):
+    """aloco_sync_host on page-locked torch CPU tensors (theta, v updated in
+    place; the replicas are read only)."""
+    import torch
+    N = global_.numel()
+    dtype = F32 if locals_[0].dtype == torch.float32 else BF16
+    if opts is None:
+        opts = default_opts()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    opts.stream = s.cuda_stream
+    M = len(locals_)
+    ptrs = (ctypes.c_void_p * M)(*[x.data_ptr() for x in locals_])
+    st = Stats()
+    rc = load().aloco_sync_host(global_.data_ptr(), momentum.data_ptr(), ptrs, N,
+                                M, dtype, H_sel, H_base, step,
+                                ctypes.byref(schedule), outer_lr, outer_beta,
+                                chunk_elems, ctypes.byref(opts), ctypes.byref(st))
+    if raise_on_error and rc not in (OK, ERR_NONFINITE):
+        raise AlocoError(rc, last_error())
+    return st.as_dict() | {"status": rc}
 
 
 def sync_int8(global_, momentum, locals_, *, parts=None, H_sel: int,

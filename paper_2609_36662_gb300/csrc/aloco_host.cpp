@@ -181,6 +181,14 @@ struct Workspace {
     size_t i8_cap = 0;
     double *host = nullptr;               // pinned readback of totals + nf
     cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+    // host-memory round (aloco_sync_host): staging slots and per-chunk totals
+    char *hs = nullptr;                   // device, grown on demand
+    size_t hs_cap = 0;
+    double *hs_host = nullptr;            // pinned per-chunk totals
+    size_t hs_host_cap = 0;               // doubles
+    cudaStream_t hs_in = nullptr, hs_out = nullptr;
+    cudaEvent_t hs_start = nullptr, hs_end = nullptr;
+    cudaEvent_t hs_loaded[3] = {}, hs_computed[3] = {}, hs_free[3] = {};
 };
 
 constexpr int kTotals = aloco::kTotalsSlots;
@@ -744,6 +752,249 @@ int aloco_int8_decode(const int8_t *codes, const float *scales, size_t N,
     return ALOCO_OK;
 }
 
+int aloco_sync_host(float *global, float *momentum, const void *const *locals,
+                    size_t N, int M, aloco_dtype dtype, int64_t H_sel,
+                    int64_t H_base, int64_t step, const aloco_schedule_t *schedule,
+                    double outer_lr, double outer_beta, size_t chunk_elems,
+                    const aloco_opts_t *opts, aloco_stats_t *stats_out) {
+    constexpr int kSlots = 3;
+    aloco_opts_t o;
+    if (opts) o = *opts; else fill_default_opts(&o);
+    aloco_stats_t local_stats;
+    aloco_stats_t *st = stats_out ? stats_out : &local_stats;
+    if (M < 1 || M > ALOCO_MAX_WORKERS)
+        return fail(ALOCO_ERR_ARG, "M = %d outside [1, %d]", M, ALOCO_MAX_WORKERS);
+    if (dtype != ALOCO_F32 && dtype != ALOCO_BF16)
+        return fail(ALOCO_ERR_ARG, "unknown replica dtype %d", (int)dtype);
+    if (o.pass != ALOCO_PASS_AUTO && o.pass != ALOCO_PASS_REGISTERS)
+        return fail(ALOCO_ERR_ARG, "the host-memory round runs the register pass; pass %d "
+                    "does not apply", o.pass);
+    if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
+    if (N > 0 && (!global || !momentum || !locals))
+        return fail(ALOCO_ERR_ARG, "NULL buffer");
+    for (int m = 0; N > 0 && m < M; ++m)
+        if (!locals[m]) return fail(ALOCO_ERR_ARG, "locals[%d] is NULL", m);
+    aloco_correction_t corr;
+    int rc = correction_impl(schedule, step, H_sel, H_base, outer_lr, outer_beta, o, &corr);
+    if (rc != ALOCO_OK) return rc;
+    std::memset(st, 0, sizeof *st);
+    st->corr = corr;
+    st->M = M;
+    st->kernel_ms = -1.f;
+    if (N == 0) {
+        t_err.clear();
+        return ALOCO_OK;
+    }
+    const size_t rsz = dtype == ALOCO_F32 ? 4 : 2;
+    {
+        std::vector<std::pair<uintptr_t, size_t>> r;
+        r.push_back({(uintptr_t)global, N * 4});
+        r.push_back({(uintptr_t)momentum, N * 4});
+        for (int m = 0; m < M; ++m) r.push_back({(uintptr_t)locals[m], N * rsz});
+        for (size_t i = 0; i < r.size(); ++i)
+            for (size_t j = i + 1; j < r.size(); ++j)
+                if (r[i].first < r[j].first + r[j].second &&
+                    r[j].first < r[i].first + r[i].second)
+                    return fail(ALOCO_ERR_ALIAS, "buffers %zu and %zu overlap", i, j);
+    }
+    if (((uintptr_t)global | (uintptr_t)momentum) & 3)
+        return fail(ALOCO_ERR_ARG, "global/momentum not 4-byte aligned");
+    for (int m = 0; m < M; ++m)
+        if ((uintptr_t)locals[m] & (rsz - 1))
+            return fail(ALOCO_ERR_ARG, "locals[%d] not %zu-byte aligned", m, rsz);
+    {
+        const void *ptrs[2 + ALOCO_MAX_WORKERS] = {global, momentum};
+        for (int m = 0; m < M; ++m) ptrs[2 + m] = locals[m];
+        for (int i = 0; i < M + 2; ++i) {
+            cudaPointerAttributes at;
+            cudaError_t e = cudaPointerGetAttributes(&at, ptrs[i]);
+            if (e != cudaSuccess) cudaGetLastError();
+            if (e != cudaSuccess || at.type != cudaMemoryTypeHost)
+                return fail(ALOCO_ERR_ARG,
+                            "buffer %d is not page-locked host memory (allocate it with "
+                            "cudaMallocHost or register it with cudaHostRegister)", i);
+        }
+    }
+    size_t chunk = chunk_elems ? chunk_elems : ((size_t)1 << 24);
+    chunk = (chunk + 7) / 8 * 8;
+    if (chunk > N) chunk = (N + 7) / 8 * 8;
+    const size_t n_chunks = (N + chunk - 1) / chunk;
+
+    int device = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    Workspace *ws = workspace_for(device);
+    std::lock_guard<std::mutex> lk(ws->mu);
+    rc = ensure_ready(ws, device);
+    if (rc != ALOCO_OK) return rc;
+
+    // streams, events and staging (grown on demand, kept until shutdown)
+    if (!ws->hs_in) {
+        e = cudaStreamCreateWithFlags(&ws->hs_in, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&ws->hs_out, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ws->hs_start, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ws->hs_end, cudaEventDisableTiming);
+        for (int k = 0; e == cudaSuccess && k < kSlots; ++k) {
+            e = cudaEventCreateWithFlags(&ws->hs_loaded[k], cudaEventDisableTiming);
+            if (e == cudaSuccess)
+                e = cudaEventCreateWithFlags(&ws->hs_computed[k], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ws->hs_free[k], cudaEventDisableTiming);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "host-round streams and events");
+    }
+    auto up256 = [](size_t b) { return (b + 255) / 256 * 256; };
+    const size_t arr4 = up256(chunk * 4), arrx = up256(chunk * rsz);
+    const size_t slot_bytes = 2 * arr4 + (size_t)M * arrx;
+    const size_t tot_bytes = n_chunks * aloco::kTotalsSlots * sizeof(double);
+    const size_t need = kSlots * slot_bytes + up256(tot_bytes);
+    if (ws->hs_cap < need) {
+        if (ws->hs) cudaFree(ws->hs);
+        ws->hs = nullptr;
+        ws->hs_cap = 0;
+        e = cudaMalloc((void **)&ws->hs, need);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(ALOCO_ERR_NOMEM, "host-round staging cudaMalloc(%zu): %s", need,
+                        cudaGetErrorString(e));
+        }
+        ws->hs_cap = need;
+    }
+    const size_t host_need = n_chunks * aloco::kTotalsSlots;
+    if (ws->hs_host_cap < host_need) {
+        if (ws->hs_host) cudaFreeHost(ws->hs_host);
+        ws->hs_host = nullptr;
+        ws->hs_host_cap = 0;
+        e = cudaMallocHost((void **)&ws->hs_host, host_need * sizeof(double));
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(ALOCO_ERR_NOMEM, "host-round read-back cudaMallocHost: %s",
+                        cudaGetErrorString(e));
+        }
+        ws->hs_host_cap = host_need;
+    }
+    double *chunk_totals = reinterpret_cast<double *>(ws->hs + kSlots * slot_bytes);
+
+    aloco::SyncArgs a;
+    std::memset(&a, 0, sizeof a);
+    split_coef(corr.inv_norm / (double)M, &a.c_hi, &a.c_lo);
+    split_coef(corr.mu_t, &a.mu_hi, &a.mu_lo);
+    split_coef(-corr.eta_out, &a.neg_eta_hi, &a.neg_eta_lo);
+    a.M = M;
+    a.partials = ws->partials;
+    a.nf_partials = ws->nf_partials;
+    a.ticket = ws->ticket;
+    a.totals = ws->totals;
+    a.nf_total = ws->nf_total;
+    a.error = ws->error;
+    const int pack = aloco::pack_elems(dtype);
+
+    cudaStream_t main_s = (cudaStream_t)o.stream;
+    auto ck = [&](cudaError_t err, const char *what) -> int {
+        if (err == cudaSuccess) return ALOCO_OK;
+        cudaStreamSynchronize(ws->hs_in);
+        cudaStreamSynchronize(ws->hs_out);
+        cudaStreamSynchronize(main_s);
+        return cuda_fail(err, what);
+    };
+    if (o.time_kernel && (rc = ck(cudaEventRecord(ws->ev0, main_s), "cudaEventRecord")))
+        return rc;
+    // the copies start after the work already queued on the caller's stream
+    if ((rc = ck(cudaEventRecord(ws->hs_start, main_s), "cudaEventRecord")) ||
+        (rc = ck(cudaStreamWaitEvent(ws->hs_in, ws->hs_start, 0), "cudaStreamWaitEvent")) ||
+        (rc = ck(cudaStreamWaitEvent(ws->hs_out, ws->hs_start, 0), "cudaStreamWaitEvent")))
+        return rc;
+    for (size_t c = 0; c < n_chunks; ++c) {
+        const int k = (int)(c % kSlots);
+        const size_t off = c * chunk;
+        const size_t n = std::min(chunk, N - off);
+        char *slot = ws->hs + k * slot_bytes;
+        float *sg = reinterpret_cast<float *>(slot);
+        float *sv = reinterpret_cast<float *>(slot + arr4);
+        char *sx = slot + 2 * arr4;
+        if (c >= (size_t)kSlots &&
+            (rc = ck(cudaStreamWaitEvent(ws->hs_in, ws->hs_free[k], 0), "cudaStreamWaitEvent")))
+            return rc;
+        rc = ck(cudaMemcpyAsync(sg, global + off, n * 4, cudaMemcpyHostToDevice, ws->hs_in),
+                "host-round copy in");
+        if (!rc)
+            rc = ck(cudaMemcpyAsync(sv, momentum + off, n * 4, cudaMemcpyHostToDevice,
+                                    ws->hs_in), "host-round copy in");
+        for (int m = 0; !rc && m < M; ++m)
+            rc = ck(cudaMemcpyAsync(sx + m * arrx,
+                                    static_cast<const char *>(locals[m]) + off * rsz, n * rsz,
+                                    cudaMemcpyHostToDevice, ws->hs_in), "host-round copy in");
+        if (!rc) rc = ck(cudaEventRecord(ws->hs_loaded[k], ws->hs_in), "cudaEventRecord");
+        if (!rc) rc = ck(cudaStreamWaitEvent(main_s, ws->hs_loaded[k], 0), "cudaStreamWaitEvent");
+        if (rc) return rc;
+
+        a.g = sg;
+        a.v = sv;
+        for (int m = 0; m < M; ++m) a.x[m] = sx + m * arrx;
+        a.n = (int64_t)n;
+        a.nvec = (int64_t)(n / pack);
+        aloco::LaunchPlan plan;
+        e = dtype == ALOCO_F32
+                ? aloco::plan_sync_f32(M, a.nvec > 0 ? a.nvec : a.n, ws->sm_count,
+                                       o.blocks_per_sm, &plan)
+                : aloco::plan_sync_bf16(M, a.nvec > 0 ? a.nvec : a.n, ws->sm_count,
+                                        o.blocks_per_sm, &plan);
+        if ((rc = ck(e, "launch plan"))) return rc;
+        a.n_tiles = plan.tiles;
+        a.stages = plan.stages;
+        void *params[] = {&a};
+        rc = ck(cudaLaunchKernel(plan.kernel, dim3(plan.grid), dim3(plan.block), params,
+                                 plan.smem, main_s), "host-round kernel launch");
+        if (!rc)
+            rc = ck(cudaMemcpyAsync(chunk_totals + c * aloco::kTotalsSlots, ws->totals,
+                                    aloco::kTotalsSlots * sizeof(double),
+                                    cudaMemcpyDeviceToDevice, main_s), "chunk totals");
+        if (!rc) rc = ck(cudaEventRecord(ws->hs_computed[k], main_s), "cudaEventRecord");
+        if (!rc)
+            rc = ck(cudaStreamWaitEvent(ws->hs_out, ws->hs_computed[k], 0), "cudaStreamWaitEvent");
+        if (!rc)
+            rc = ck(cudaMemcpyAsync(global + off, sg, n * 4, cudaMemcpyDeviceToHost, ws->hs_out),
+                    "host-round copy out");
+        if (!rc)
+            rc = ck(cudaMemcpyAsync(momentum + off, sv, n * 4, cudaMemcpyDeviceToHost,
+                                    ws->hs_out), "host-round copy out");
+        if (!rc) rc = ck(cudaEventRecord(ws->hs_free[k], ws->hs_out), "cudaEventRecord");
+        if (rc) return rc;
+    }
+    rc = ck(cudaMemcpyAsync(ws->hs_host, chunk_totals, tot_bytes, cudaMemcpyDeviceToHost, main_s),
+            "statistics readback");
+    if (!rc) rc = ck(cudaEventRecord(ws->hs_end, ws->hs_out), "cudaEventRecord");
+    if (!rc) rc = ck(cudaStreamWaitEvent(main_s, ws->hs_end, 0), "cudaStreamWaitEvent");
+    if (!rc && o.time_kernel) rc = ck(cudaEventRecord(ws->ev1, main_s), "cudaEventRecord");
+    if (rc) return rc;
+    if ((rc = ck(cudaStreamSynchronize(main_s), "host round"))) return rc;
+
+    // totals of the chunks, added in chunk order
+    double tot[aloco::kTotalsSlots] = {};
+    unsigned long long nf = 0;
+    for (size_t c = 0; c < n_chunks; ++c) {
+        const double *t = ws->hs_host + c * aloco::kTotalsSlots;
+        for (int m = 0; m <= M; ++m) tot[m] += t[m];
+        unsigned long long nfc;
+        std::memcpy(&nfc, t + aloco::kNfSlot, sizeof nfc);
+        nf += nfc;
+    }
+    finalize_stats(tot, nf, M, o.eps, 1.0 / ((double)M * (double)M), st);
+    st->grid = (int)n_chunks;
+    st->pass_used = ALOCO_PASS_REGISTERS;
+    if (o.time_kernel) {
+        float ms = -1.f;
+        if (cudaEventElapsedTime(&ms, ws->ev0, ws->ev1) == cudaSuccess)
+            st->kernel_ms = ms;
+        else
+            cudaGetLastError();
+    }
+    if (st->nonfinite > 0 || !std::isfinite(st->D) || !std::isfinite(st->C))
+        return fail(ALOCO_ERR_NONFINITE, "round produced %lld non-finite elements (D=%g, C=%g)",
+                    (long long)st->nonfinite, st->D, st->C);
+    t_err.clear();
+    return ALOCO_OK;
+}
+
 void aloco_adamw_default_cfg(aloco_adamw_cfg_t *cfg) {
     if (!cfg) return;
     std::memset(cfg, 0, sizeof *cfg);
@@ -943,6 +1194,22 @@ void aloco_shutdown(void) {
         if (ws->i8) cudaFree(ws->i8);
         ws->i8 = nullptr;
         ws->i8_cap = 0;
+        if (ws->hs) cudaFree(ws->hs);
+        if (ws->hs_host) cudaFreeHost(ws->hs_host);
+        ws->hs = nullptr;
+        ws->hs_cap = 0;
+        ws->hs_host = nullptr;
+        ws->hs_host_cap = 0;
+        cudaEvent_t *evs[] = {&ws->hs_start, &ws->hs_end};
+        for (cudaEvent_t *ev : evs)
+            if (*ev) cudaEventDestroy(*ev), *ev = nullptr;
+        for (int k = 0; k < 3; ++k) {
+            for (cudaEvent_t *ev : {&ws->hs_loaded[k], &ws->hs_computed[k], &ws->hs_free[k]})
+                if (*ev) cudaEventDestroy(*ev), *ev = nullptr;
+        }
+        if (ws->hs_in) cudaStreamDestroy(ws->hs_in);
+        if (ws->hs_out) cudaStreamDestroy(ws->hs_out);
+        ws->hs_in = ws->hs_out = nullptr;
         ws->ev0 = ws->ev1 = nullptr;
         ws->host = nullptr;
         ws->dev = nullptr;
