@@ -118,9 +118,9 @@ typedef enum {
  * The INT8-communicated round (aloco_sync_int8) has two forms of its own:
  *   INT8_SPLIT a block-scale kernel, then an apply kernel that reads the
  *              replicas again (any M <= 16);
- *   INT8_FUSED one kernel whose threads hold their replica values in
- *              registers, reading every replica once (bf16 M <= 8, fp32
- *              M <= 4; ALOCO_ERR_ARG otherwise);
+ *   INT8_FUSED one kernel that stages each block of theta, v and the
+ *              replicas in shared memory, reading every replica once
+ *              (M <= 8; ALOCO_ERR_ARG otherwise);
  *   AUTO       the form measured faster on GB300 for (M, dtype).
  * aloco_sync / aloco_sync_ex reject the INT8 values and aloco_sync_int8 the
  * REGISTERS / BULK_COPY values with ALOCO_ERR_ARG. */

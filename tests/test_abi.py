@@ -247,7 +247,7 @@ def test_pass_values_are_checked_against_the_round(lib):
                                    ctypes.byref(st))
     for p in (A.PASS_REGISTERS, A.PASS_BULK_COPY):
         assert int8(2, A.F32, p) == A.ERR_ARG
-    assert int8(5, A.F32, A.PASS_INT8_FUSED) == A.ERR_ARG
+    assert int8(9, A.F32, A.PASS_INT8_FUSED) == A.ERR_ARG
     assert int8(9, A.BF16, A.PASS_INT8_FUSED) == A.ERR_ARG
     assert "fused" in A.last_error()
     # accepted combinations get past argument checks (no device here)

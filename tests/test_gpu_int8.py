@@ -9,7 +9,7 @@ import oracle as O
 from paper_2609_36662_gb300 import aloco as A
 from paper_2609_36662_gb300 import workloads as W
 
-from _parity import (assert_bf16_replica, assert_corr, assert_field,
+from _parity import (RTOL_STAT, assert_bf16_replica, assert_corr, assert_field,
                      assert_stats, gpu_inputs, oracle_corr, schedule_pair,
                      to_numpy_bits)
 
@@ -94,7 +94,7 @@ def _compare(w, st, corr, orc, g, v, xs):
 
 
 def _fits_fused(dt, M):
-    return M <= (8 if dt == "bf16" else 4)
+    return M <= 8
 
 
 FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
@@ -106,7 +106,7 @@ FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
 @pytest.mark.parametrize("parts_name", ["one_part", "ragged", "llama_like"])
 def test_int8_round_matches_oracle(dt, M, parts_name, form):
     if form == "fused" and not _fits_fused(dt, M):
-        pytest.skip("the fused form holds bf16 M <= 8, fp32 M <= 4")
+        pytest.skip("the fused form holds M <= 8")
     parts = PARTS[parts_name]
     N = sum(parts) if parts else 5 * 4096 + 333
     w = W.small(N, M, dt, seed=40 + M)
@@ -122,12 +122,13 @@ def test_int8_round_matches_oracle(dt, M, parts_name, form):
     _compare(w, st, corr, orc, g, v, xs)
 
 
-@pytest.mark.parametrize("dt,M", [("f32", 1), ("f32", 4), ("bf16", 2),
+@pytest.mark.parametrize("dt,M", [("f32", 1), ("f32", 4), ("f32", 7), ("bf16", 2),
                                   ("bf16", 5), ("bf16", 8)])
 def test_int8_forms_agree_bit_for_bit(dt, M):
     """The fused and the split form take the same decisions in the same
     arithmetic: theta', v' and the replicas are bit-identical; the
-    statistics differ at most by the order of their fp64 sums."""
+    statistics agree within the statistics tolerance (the forms group each
+    thread's fp32 partial energies differently)."""
     parts = PARTS["llama_like"]
     w = W.small(sum(parts), M, dt, seed=70 + M)
     sa, _ = schedule_pair(w.schedule)
@@ -146,7 +147,7 @@ def test_int8_forms_agree_bit_for_bit(dt, M):
     for a, b in zip(x1, x2):
         assert torch.equal(a, b)
     for key in ("D", "C", "mean_sq_norm"):
-        assert s1[key] == pytest.approx(s2[key], rel=1e-12), key
+        assert s1[key] == pytest.approx(s2[key], rel=RTOL_STAT), key
     assert s1["nonfinite"] == s2["nonfinite"] == 0
 
 
@@ -154,8 +155,8 @@ def test_int8_auto_form():
     """AUTO takes the fused form wherever it fits, the split form beyond."""
     for dt, M, want in (("bf16", 8, A.PASS_INT8_FUSED),
                         ("bf16", 9, A.PASS_INT8_SPLIT),
-                        ("f32", 4, A.PASS_INT8_FUSED),
-                        ("f32", 5, A.PASS_INT8_SPLIT)):
+                        ("f32", 8, A.PASS_INT8_FUSED),
+                        ("f32", 9, A.PASS_INT8_SPLIT)):
         w = W.small(3 * 4096 + 5, M, dt, seed=3)
         g, v, xs = gpu_inputs(w)
         sa, _ = schedule_pair(w.schedule)
