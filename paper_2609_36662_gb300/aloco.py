@@ -36,7 +36,8 @@ EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
            "aloco_int8_decode", "aloco_adamw_default_cfg", "aloco_adamw_step",
            "aloco_ctrl_default_cfg", "aloco_ctrl_init", "aloco_select_interval",
            "aloco_ctrl_state_bytes", "aloco_ctrl_save", "aloco_ctrl_load",
-           "aloco_last_error", "aloco_shutdown", "aloco_version")
+           "aloco_test_stall_tile", "aloco_last_error", "aloco_shutdown",
+           "aloco_version")
 
 CTRL_HISTORY = 16
 ASSESS_NONE, ASSESS_SUPPORTED, ASSESS_CONSISTENT, ASSESS_MODERATE, \
@@ -210,6 +211,8 @@ def load():
     lib.aloco_adamw_step.restype = i32
     lib.aloco_sync_host.argtypes = sync_args + [ctypes.c_size_t, P(Opts), P(Stats)]
     lib.aloco_sync_host.restype = i32
+    lib.aloco_test_stall_tile.argtypes = [i64]
+    lib.aloco_test_stall_tile.restype = None
     lib.aloco_int8_num_blocks.argtypes = [vp, i32]
     lib.aloco_int8_num_blocks.restype = i64
     lib.aloco_int8_encode.argtypes = [vp, ctypes.c_size_t, vp, i32, vp, vp, vp,
@@ -552,3 +555,9 @@ def adamw_step(params, grads, exp_avg, exp_avg_sq, cfg: AdamwCfg,
     if st is None:
         return rc if not raise_on_error else None
     return st.as_dict() | {"status": rc}
+
+
+def test_stall_tile(tile: int):
+    """Testing only: the next bulk-copy round on this thread skips the copies
+    of one tile, so that its bounded wait runs out (aloco_test_stall_tile)."""
+    load().aloco_test_stall_tile(int(tile))

@@ -276,6 +276,10 @@ GetAddressRangeFn address_range_fn() {
 
 // Helpers with external linkage: also used by the allocation-free entry
 // point (aloco_noalloc.cu).
+// Testing hook of aloco_test_stall_tile: consumed by the calling thread's
+// next bulk-copy round.
+thread_local int64_t t_test_stall_tile1 = 0;
+
 namespace aloco {
 
 bool use_int8_fused(int pass, int M, aloco_dtype dtype) {
@@ -579,6 +583,10 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     a.n_tiles = plan.tiles;
     a.stages = plan.stages;
     a.error = ws->error;
+    if (tma) {
+        a.test_stall_tile1 = t_test_stall_tile1;
+        t_test_stall_tile1 = 0;
+    }
     if (plan.grid > ws->max_grid)
         return fail(ALOCO_ERR_CUDA, "grid %d exceeds workspace %d", plan.grid,
                     ws->max_grid);
@@ -1174,6 +1182,8 @@ int aloco_adamw_step(void *const *params, const void *const *grads,
     t_err.clear();
     return ALOCO_OK;
 }
+
+void aloco_test_stall_tile(int64_t tile) { t_test_stall_tile1 = tile >= 0 ? tile + 1 : 0; }
 
 const char *aloco_last_error(void) { return t_err.c_str(); }
 

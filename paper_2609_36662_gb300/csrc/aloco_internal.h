@@ -38,6 +38,8 @@ struct SyncArgs {
     int64_t n_tiles;                // whole tiles of kTmaConsumers packs
     int stages;                     // depth of the shared-memory ring
     unsigned int *error;            // set to 1 if a pipeline wait timed out
+    int64_t test_stall_tile1;       // testing only: 1 + the index of a tile whose
+                                    // copies the producer skips (0 = none)
 };
 
 // Slots of the totals block read back after a round (8 bytes each): M + 1

@@ -190,6 +190,12 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
                 }
                 if (*abort_v) break;
                 const int64_t t = b + j * G;
+                if (a.test_stall_tile1 != 0 && t == a.test_stall_tile1 - 1) {
+                    // testing only: this stage's full barrier never completes,
+                    // so the consumers' bounded wait runs out
+                    issued = j + 1;
+                    continue;
+                }
                 const uint32_t st = ring + (uint32_t)s * kStage;
                 const uint32_t fb = smem_addr(&full_bar[s]);
                 mbar_arrive_expect_tx(fb, kStage);
