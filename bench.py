@@ -757,6 +757,86 @@ def run_adamw(args, w):
     return 0
 
 
+# ---------------------------------------------------- whole-interval mode
+
+INTERVAL_METRIC = ("inner steps/s of whole AutoLoCo intervals (H AdamW steps on "
+                   "all M replicas, the outer round and the controller) and the "
+                   "outer round's share of the interval time")
+
+
+def run_interval(args, w):
+    """Whole intervals on one GPU: the C4 recipe's controller (H_base 500 in
+    [250, 750], q_H 50) picks each interval's horizon; an interval is that
+    many aloco_adamw_step calls (the same synthetic gradients every step),
+    then aloco_sync with the statistics, then aloco_select_interval.  Each
+    interval's inner loop and round are timed with CUDA events."""
+    import torch
+    from paper_2609_36662_gb300 import aloco as A
+    from paper_2609_36662_gb300 import workloads as W
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", torch.cuda.current_device())
+    A.load()
+    xs, gs, m1, m2 = adamw_inputs(w, device)
+    g = W.make_global(w, device)
+    v = W.make_momentum(w, device)
+    for x in xs:
+        x.copy_(g.to(x.dtype))
+    sched = A.Schedule.make(0, 4e-4, 4e-5, 1000, 50_000)
+    ctrl = A.Controller(500, 250, 750, 50, 1000, sched)
+    stream = torch.cuda.Stream(device)
+    opts = A.default_opts()
+    step = 2000                      # past the warm-up of the schedule
+    inner_ms, round_ms, hs = [], [], []
+    for k in range(args.warmup + args.steps):
+        h = ctrl.decision.H_step
+        e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        e0.record(stream)
+        for i in range(h):
+            A.adamw_step(xs, gs, m1, m2,
+                         A.adamw_cfg(lr=A.inner_lr_accum(sched, step + i, 1),
+                                     step=step + i + 1),
+                         opts=opts, stream=stream, want_stats=False)
+        e1.record(stream)
+        st = A.sync(g, v, xs, H_sel=h, H_base=ctrl.decision.H_ref_step,
+                    step=step, schedule=sched, outer_lr=0.7, outer_beta=0.9,
+                    opts=opts, stream=stream, raise_on_error=False)
+        ctrl.observe(st["D"], st["C"], st["corr"]["lam_sel"], 1024.0 * h, h,
+                     step + h)
+        e2.record(stream)
+        e2.synchronize()
+        step += h
+        if k >= args.warmup:
+            inner_ms.append(e0.elapsed_time(e1))
+            round_ms.append(e1.elapsed_time(e2))
+            hs.append(h)
+    tot_ms = sum(inner_ms) + sum(round_ms)
+    tot_ms = reduce_max(tot_ms, world, device)
+    value = job_value(float(sum(hs)), tot_ms / 1e3, world)
+    if rank == 0:
+        line = {
+            "metric": INTERVAL_METRIC, "value": value, "unit": "inner steps/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": tot_ms / len(hs), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded replicas, fixed synthetic gradients)",
+            "config": dict(adamw_config(w), mode="interval",
+                           controller="C4 recipe: H_base 500 in [250, 750], "
+                                      "q_H 50, cosine 4e-4 -> 4e-5, warm-up 1000"),
+            "intervals": [{"H": h, "inner_ms": a, "round_ms": b}
+                          for h, a, b in zip(hs, inner_ms, round_ms)],
+            "round_share": sum(round_ms) / (sum(inner_ms) + sum(round_ms)),
+            "ms_per_inner_step": sum(inner_ms) / sum(hs),
+            "gpu_launches": 2 * sum(hs) + len(hs),
+            "cpu_baseline": None, "e2e": None,
+        }
+        print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     p.add_argument("--gpus", type=int, default=1)
@@ -777,9 +857,10 @@ def main(argv=None):
     p.add_argument("--comm", choices=["fp32", "int8"], default="fp32",
                    help="int8: the round with INT8-communicated "
                         "pseudo-gradients (App. G.1)")
-    p.add_argument("--mode", choices=["round", "adamw"], default="round",
-                   help="adamw: time the workers' inner AdamW step instead "
-                        "of the outer round")
+    p.add_argument("--mode", choices=["round", "adamw", "interval"],
+                   default="round",
+                   help="adamw: time the workers' inner AdamW step; interval: "
+                        "whole intervals (inner steps, round, controller)")
     p.add_argument("--list", action="store_true")
     args = p.parse_args(argv)
     table = workloads_by_name()
@@ -797,6 +878,13 @@ def main(argv=None):
     if args.mode == "adamw":
         return (run_adamw_reference(args, w) if args.impl == "reference"
                 else run_adamw(args, w))
+    if args.mode == "interval":
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable":
+                              "the interval mode has no reference arm; "
+                              "--mode adamw and --mode round do"}))
+            return 0
+        return run_interval(args, w)
     if args.impl == "reference":
         return run_reference(args, w)
     return run_cuda(args, w)
