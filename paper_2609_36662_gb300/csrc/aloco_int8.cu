@@ -362,7 +362,9 @@ template <bool BF16>
 cudaError_t round_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
                          unsigned *bmax, double *e_rows, int max_grid,
                          cudaStream_t stream, int *grid_out) {
-    static int occ = 0;
+    static PerDevice cache;
+    const int dev = PerDevice::device();
+    int occ = cache.get(dev);
     if (occ == 0) {
         int b1 = 0, b2 = 0;
         cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
@@ -373,6 +375,7 @@ cudaError_t round_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
         if (e != cudaSuccess) return e;
         occ = b1 < b2 ? b1 : b2;
         if (occ < 1) occ = 1;
+        cache.set(dev, occ);
     }
     const int64_t nblocks = P.blk[P.n_parts];
     int64_t grid = (int64_t)sm_count * occ;

@@ -502,8 +502,9 @@ cudaError_t fused_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
                          int max_grid, cudaStream_t stream, int *grid_out) {
     constexpr int T = fused_threads<M, BF16>();
     constexpr size_t smem = n_bufs<M, BF16, T>() * stage_bytes<M, BF16, T>();
-    static std::atomic<int> occ_cache{0};
-    int occ = occ_cache.load(std::memory_order_relaxed);
+    static PerDevice occ_cache;  // attribute set-up and occupancy, per device
+    const int dev = PerDevice::device();
+    int occ = occ_cache.get(dev);
     if (occ == 0) {
         cudaError_t e = cudaFuncSetAttribute(int8_fused_kernel<M, BF16, T>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -513,7 +514,7 @@ cudaError_t fused_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
                 &occ, int8_fused_kernel<M, BF16, T>, T, smem);
         if (e != cudaSuccess) return e;
         if (occ < 1) occ = 1;
-        occ_cache.store(occ, std::memory_order_relaxed);
+        occ_cache.set(dev, occ);
     }
     const int64_t nblocks = P.blk[P.n_parts];
     int64_t grid = (int64_t)sm_count * occ;

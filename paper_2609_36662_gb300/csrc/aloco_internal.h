@@ -5,9 +5,32 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/aloco.h"
 
 namespace aloco {
+
+// A value computed once per device and kept for the process: function
+// attributes and occupancy belong to a device's context, so launch set-up is
+// cached per device (zero = not yet computed).  Devices beyond kMaxDevices
+// are not cached and recompute every time.
+constexpr int kMaxDevices = 64;
+struct PerDevice {
+    std::atomic<int> v[kMaxDevices];
+    static int device() {
+        int d = -1;
+        if (cudaGetDevice(&d) != cudaSuccess) {
+            cudaGetLastError();
+            return -1;
+        }
+        return d >= 0 && d < kMaxDevices ? d : -1;
+    }
+    int get(int d) const { return d >= 0 ? v[d].load(std::memory_order_acquire) : 0; }
+    void set(int d, int x) {
+        if (d >= 0) v[d].store(x, std::memory_order_release);
+    }
+};
 
 // Threads per block of the fused pass.
 constexpr int kBlock = 256;

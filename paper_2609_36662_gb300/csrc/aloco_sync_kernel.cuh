@@ -462,8 +462,10 @@ constexpr int tuned_blocks_per_sm(int M) {
 template <int MT, bool BF16>
 cudaError_t plan_one(int64_t work_items, int sm_count, int M, int request,
                      LaunchPlan *plan) {
-    static int occupancy = 0;  // per instance, computed once
+    static PerDevice cache;  // per instance and device, computed once
     const void *fn = reinterpret_cast<const void *>(&sync_kernel<MT, BF16>);
+    const int dev = PerDevice::device();
+    int occupancy = cache.get(dev);
     if (occupancy == 0) {
         int b = 0;
         cudaError_t e =
@@ -471,6 +473,7 @@ cudaError_t plan_one(int64_t work_items, int sm_count, int M, int request,
                                                           kBlock, 0);
         if (e != cudaSuccess) return e;
         occupancy = b > 0 ? b : 1;
+        cache.set(dev, occupancy);
     }
     int blocks_per_sm = request > 0 ? request : tuned_blocks_per_sm<BF16>(M);
     if (blocks_per_sm <= 0 || blocks_per_sm > occupancy) blocks_per_sm = occupancy;

@@ -312,16 +312,17 @@ constexpr int tma_stages(int M, int smem_budget) {
 template <int MT, bool BF16>
 cudaError_t plan_tma_one(int64_t nvec, int sm_count, int smem_budget,
                          LaunchPlan *plan) {
-    static bool configured = false;
+    static PerDevice configured;  // the shared-memory attribute, per device
     const int stages = tma_stages<BF16>(MT, smem_budget);
     if (stages < 2) return cudaErrorInvalidValue;
     const int smem = stages * (int)tma_stage_bytes<BF16>(MT);
-    if (!configured) {
+    const int dev = PerDevice::device();
+    if (!configured.get(dev)) {
         cudaError_t e = cudaFuncSetAttribute(
             sync_tma_kernel<MT, BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
             smem_budget);
         if (e != cudaSuccess) return e;
-        configured = true;
+        configured.set(dev, 1);
     }
     const int64_t tiles = nvec / kTmaConsumers;
     plan->kernel = reinterpret_cast<const void *>(&sync_tma_kernel<MT, BF16>);
