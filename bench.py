@@ -674,12 +674,19 @@ def run_adamw(args, w):
     ev = [(torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True))
           for _ in range(args.warmup + args.steps)]
+    # "given": the gradients' norms are known to the caller (taken once from
+    # a regular step here), and the one-pass aloco_adamw_step_normed runs
+    norms = None
+    if args.adamw_norms == "given":
+        norms = A.adamw_step(xs, gs, m1, m2, A.adamw_cfg(lr=ADAMW_LR,
+                                                         step=ADAMW_STEP0),
+                             opts=opts, stream=stream)["grad_norm"]
 
     def one_step(k):
         cfg = A.adamw_cfg(lr=ADAMW_LR, step=ADAMW_STEP0 + k)
         ev[k][0].record(stream)
         A.adamw_step(xs, gs, m1, m2, cfg, opts=opts, stream=stream,
-                     want_stats=False)
+                     want_stats=False, grad_norms=norms)
         ev[k][1].record(stream)
 
     for k in range(args.warmup):
@@ -744,13 +751,17 @@ def run_adamw(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
                          "unit": "GB/s", "frac": achieved / peak,
                          "peak_source": peak_kind,
-                         "traffic": recorded_traffic(w.name, "adamw_kernels"),
-                         "kernel": "adamw_kernels",
+                         "traffic": (recorded_traffic(w.name, "adamw_kernels")
+                                     if norms is None else None),
+                         "kernel": ("adamw_kernels" if norms is None
+                                    else "adamw_update_kernel"),
                          "algorithmic_bytes_per_launch": adamw_bytes(w)},
             "grad_norms": st["grad_norm"], "clip": st["clip"],
             "cpu_baseline": cpu_baseline, "e2e": e2e,
-            # two kernels per step: gradient norms, then the update
-            "gpu_launches": 2 * args.steps,
+            # two kernels per step (gradient norms, then the update), or the
+            # update alone with given norms
+            "gpu_launches": (2 if norms is None else 1) * args.steps,
+            "grad_norms_source": "computed" if norms is None else "given",
             "clocks": clocks.summary(),
         }
         print(json.dumps(line), flush=True)
@@ -861,6 +872,10 @@ def main(argv=None):
                    default="round",
                    help="adamw: time the workers' inner AdamW step; interval: "
                         "whole intervals (inner steps, round, controller)")
+    p.add_argument("--adamw-norms", choices=["computed", "given"],
+                   default="computed",
+                   help="--mode adamw: compute the clipping norms (two "
+                        "passes) or take them from the caller (one pass)")
     p.add_argument("--list", action="store_true")
     args = p.parse_args(argv)
     table = workloads_by_name()

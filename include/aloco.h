@@ -379,6 +379,21 @@ int aloco_adamw_step(void *const *params, const void *const *grads,
                      const aloco_adamw_cfg_t *cfg, const aloco_opts_t *opts,
                      aloco_adamw_stats_t *stats_out);
 
+/* aloco_adamw_step for callers that already have the replicas' gradient
+ * norms (for instance from the backward pass that produced the gradients):
+ * grad_norms is a host array of M finite, non-negative values ||g_m||.  The
+ * clipping factors are formed from them on the host, exactly as
+ * aloco_adamw_step forms them from its own norms, and only the update pass
+ * runs, reading each gradient once.  stats_out (optional) reports the given
+ * norms and the factors applied; with stats_out == NULL the call only
+ * enqueues.  Other arguments and errors as aloco_adamw_step. */
+int aloco_adamw_step_normed(void *const *params, const void *const *grads,
+                            float *const *exp_avg, float *const *exp_avg_sq,
+                            size_t N, int M, aloco_dtype param_dtype,
+                            aloco_dtype grad_dtype, const aloco_adamw_cfg_t *cfg,
+                            const double *grad_norms, const aloco_opts_t *opts,
+                            aloco_adamw_stats_t *stats_out);
+
 /* ------------------------------------------------------------------------
  * Interval controller (Sec. 3.1; App. A).  Host-only and scalar: after each
  * completed interval it takes that interval's D_t, C_t, accumulated inner

@@ -34,6 +34,7 @@ EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
            "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc", "aloco_sync_host",
            "aloco_sync_int8", "aloco_int8_num_blocks", "aloco_int8_encode",
            "aloco_int8_decode", "aloco_adamw_default_cfg", "aloco_adamw_step",
+           "aloco_adamw_step_normed",
            "aloco_ctrl_default_cfg", "aloco_ctrl_init", "aloco_select_interval",
            "aloco_ctrl_state_bytes", "aloco_ctrl_save", "aloco_ctrl_load",
            "aloco_test_stall_tile", "aloco_last_error", "aloco_shutdown",
@@ -209,6 +210,10 @@ def load():
                                      i32, i32, P(AdamwCfg), P(Opts),
                                      P(AdamwStats)]
     lib.aloco_adamw_step.restype = i32
+    lib.aloco_adamw_step_normed.argtypes = [vp, vp, vp, vp, ctypes.c_size_t, i32,
+                                            i32, i32, P(AdamwCfg), vp, P(Opts),
+                                            P(AdamwStats)]
+    lib.aloco_adamw_step_normed.restype = i32
     lib.aloco_sync_host.argtypes = sync_args + [ctypes.c_size_t, P(Opts), P(Stats)]
     lib.aloco_sync_host.restype = i32
     lib.aloco_test_stall_tile.argtypes = [i64]
@@ -524,11 +529,13 @@ def adamw_cfg(**kw) -> AdamwCfg:
 
 def adamw_step(params, grads, exp_avg, exp_avg_sq, cfg: AdamwCfg,
                opts: Optional[Opts] = None, stream=None, want_stats=True,
-               raise_on_error=True):
+               raise_on_error=True, grad_norms=None):
     """One AdamW step on every replica, in place (lists of torch CUDA tensors
-    of one device: params and grads fp32 or bf16, moments fp32).  Returns the
-    per-replica gradient norms and clipping factors (want_stats), else None
-    without waiting for the GPU."""
+    of one device: params and grads fp32 or bf16, moments fp32).  With
+    grad_norms (M floats, the gradients' norms) the step takes them instead
+    of computing them (aloco_adamw_step_normed).  Returns the per-replica
+    gradient norms and clipping factors (want_stats), else None without
+    waiting for the GPU."""
     import torch
     M = len(params)
     if not (len(grads) == len(exp_avg) == len(exp_avg_sq) == M):
@@ -546,10 +553,17 @@ def adamw_step(params, grads, exp_avg, exp_avg_sq, cfg: AdamwCfg,
         return (ctypes.c_void_p * M)(*[t.data_ptr() for t in ts])
     st = AdamwStats() if want_stats else None
     with torch.cuda.device(params[0].device):
-        rc = load().aloco_adamw_step(arr(params), arr(grads), arr(exp_avg),
-                                     arr(exp_avg_sq), N, M, pdt, gdt,
-                                     ctypes.byref(cfg), ctypes.byref(opts),
-                                     ctypes.byref(st) if st is not None else None)
+        if grad_norms is None:
+            rc = load().aloco_adamw_step(arr(params), arr(grads), arr(exp_avg),
+                                         arr(exp_avg_sq), N, M, pdt, gdt,
+                                         ctypes.byref(cfg), ctypes.byref(opts),
+                                         ctypes.byref(st) if st is not None else None)
+        else:
+            norms = (ctypes.c_double * M)(*[float(x) for x in grad_norms])
+            rc = load().aloco_adamw_step_normed(
+                arr(params), arr(grads), arr(exp_avg), arr(exp_avg_sq), N, M, pdt,
+                gdt, ctypes.byref(cfg), norms, ctypes.byref(opts),
+                ctypes.byref(st) if st is not None else None)
     if raise_on_error and rc != OK:
         raise AlocoError(rc, last_error())
     if st is None:

@@ -11,6 +11,8 @@
 //                then a fixed shuffle tree) into ||g_m|| and the clipping
 //                factor c_m, so all blocks agree without a device-wide sync;
 //                then it streams x, g, m, v of replica m and writes x, m, v.
+// When the caller supplies the norms (aloco_adamw_step_normed) the factors
+// arrive with the arguments and only the update pass runs.
 // Both passes are deterministic: the partition depends only on the grid.
 // The update reads each array once; the gradient is read a second time by
 // the norm pass, which clipping needs before any element can move.
@@ -130,7 +132,9 @@ __global__ void __launch_bounds__(kBlock)
     adamw_update_kernel(const __grid_constant__ AdamArgs a) {
     const int m = blockIdx.y;
     __shared__ float s_clip;
-    if (threadIdx.x < 32) {
+    if (a.given) {
+        if (threadIdx.x == 0) s_clip = a.clip[m];
+    } else if (threadIdx.x < 32) {
         double s = 0.0;
         for (int b = threadIdx.x; b < a.g1; b += 32) s += a.partials[(int64_t)m * a.g1 + b];
 #pragma unroll
@@ -198,9 +202,11 @@ namespace {
 template <bool PBF16, bool GBF16>
 cudaError_t adamw_launch(const AdamArgs &a, int g2, cudaStream_t stream) {
     const dim3 block(kBlock);
-    adamw_norm_kernel<GBF16><<<dim3(a.g1, a.M), block, 0, stream>>>(a);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    if (!a.given) {
+        adamw_norm_kernel<GBF16><<<dim3(a.g1, a.M), block, 0, stream>>>(a);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
     adamw_update_kernel<PBF16, GBF16><<<dim3(g2, a.M), block, 0, stream>>>(a);
     return cudaGetLastError();
 }

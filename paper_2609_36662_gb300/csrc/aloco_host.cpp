@@ -1003,6 +1003,31 @@ int aloco_sync_host(float *global, float *momentum, const void *const *locals,
     return ALOCO_OK;
 }
 
+static int adamw_impl(void *const *params, const void *const *grads,
+                      float *const *exp_avg, float *const *exp_avg_sq, size_t N,
+                      int M, aloco_dtype param_dtype, aloco_dtype grad_dtype,
+                      const aloco_adamw_cfg_t *cfg, const double *norms_in,
+                      const aloco_opts_t *opts, aloco_adamw_stats_t *stats_out);
+
+int aloco_adamw_step(void *const *params, const void *const *grads,
+                     float *const *exp_avg, float *const *exp_avg_sq, size_t N,
+                     int M, aloco_dtype param_dtype, aloco_dtype grad_dtype,
+                     const aloco_adamw_cfg_t *cfg, const aloco_opts_t *opts,
+                     aloco_adamw_stats_t *stats_out) {
+    return adamw_impl(params, grads, exp_avg, exp_avg_sq, N, M, param_dtype, grad_dtype,
+                      cfg, nullptr, opts, stats_out);
+}
+
+int aloco_adamw_step_normed(void *const *params, const void *const *grads,
+                            float *const *exp_avg, float *const *exp_avg_sq, size_t N,
+                            int M, aloco_dtype param_dtype, aloco_dtype grad_dtype,
+                            const aloco_adamw_cfg_t *cfg, const double *grad_norms,
+                            const aloco_opts_t *opts, aloco_adamw_stats_t *stats_out) {
+    if (!grad_norms) return fail(ALOCO_ERR_ARG, "NULL grad_norms");
+    return adamw_impl(params, grads, exp_avg, exp_avg_sq, N, M, param_dtype, grad_dtype,
+                      cfg, grad_norms, opts, stats_out);
+}
+
 void aloco_adamw_default_cfg(aloco_adamw_cfg_t *cfg) {
     if (!cfg) return;
     std::memset(cfg, 0, sizeof *cfg);
@@ -1015,11 +1040,11 @@ void aloco_adamw_default_cfg(aloco_adamw_cfg_t *cfg) {
     cfg->step = 1;
 }
 
-int aloco_adamw_step(void *const *params, const void *const *grads,
-                     float *const *exp_avg, float *const *exp_avg_sq, size_t N,
-                     int M, aloco_dtype param_dtype, aloco_dtype grad_dtype,
-                     const aloco_adamw_cfg_t *cfg, const aloco_opts_t *opts,
-                     aloco_adamw_stats_t *stats_out) {
+static int adamw_impl(void *const *params, const void *const *grads,
+                      float *const *exp_avg, float *const *exp_avg_sq, size_t N,
+                      int M, aloco_dtype param_dtype, aloco_dtype grad_dtype,
+                      const aloco_adamw_cfg_t *cfg, const double *norms_in,
+                      const aloco_opts_t *opts, aloco_adamw_stats_t *stats_out) {
     aloco_opts_t o;
     if (opts) o = *opts; else fill_default_opts(&o);
     if (!cfg) return fail(ALOCO_ERR_ARG, "NULL cfg");
@@ -1042,6 +1067,22 @@ int aloco_adamw_step(void *const *params, const void *const *grads,
     if (!std::isfinite(c.max_grad_norm))
         return fail(ALOCO_ERR_ARG, "max_grad_norm must be finite");
     if (c.step < 1) return fail(ALOCO_ERR_ARG, "step = %lld must be >= 1", (long long)c.step);
+    // clipping factors from given norms: the update kernel's formula, in
+    // the same double arithmetic
+    double given_clip[ALOCO_MAX_WORKERS];
+    if (norms_in) {
+        for (int m = 0; m < M; ++m) {
+            const double nm = norms_in[m];
+            if (!(std::isfinite(nm) && nm >= 0.0))
+                return fail(ALOCO_ERR_ARG, "grad_norms[%d] = %g must be finite and >= 0", m, nm);
+            double cf = 1.0;
+            if (c.max_grad_norm > 0.0) {
+                cf = c.max_grad_norm / (nm + 1e-6);
+                if (cf > 1.0) cf = 1.0;
+            }
+            given_clip[m] = cf;
+        }
+    }
     if (o.blocks_per_sm < 0)
         return fail(ALOCO_ERR_ARG, "blocks_per_sm = %d must be >= 0", o.blocks_per_sm);
     if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
@@ -1056,7 +1097,10 @@ int aloco_adamw_step(void *const *params, const void *const *grads,
     std::memset(st, 0, sizeof *st);
     st->M = M;
     st->kernel_ms = -1.f;
-    for (int m = 0; m < M; ++m) st->clip[m] = 1.0;
+    for (int m = 0; m < M; ++m) {
+        st->clip[m] = norms_in ? given_clip[m] : 1.0;
+        if (norms_in) st->grad_norm[m] = norms_in[m];
+    }
     if (N == 0) {
         t_err.clear();
         return ALOCO_OK;
@@ -1139,6 +1183,10 @@ int aloco_adamw_step(void *const *params, const void *const *grads,
     a.max_norm = c.max_grad_norm;
     a.partials = ws->adam;
     a.out = ws->adam + ws->max_grid;
+    if (norms_in) {
+        a.given = 1;
+        for (int m = 0; m < M; ++m) a.clip[m] = (float)given_clip[m];
+    }
 
     // norm pass: up to the workspace's max_grid blocks over all workers;
     // update pass: SMs x blocks_per_sm blocks (default 4) over all workers
@@ -1162,7 +1210,17 @@ int aloco_adamw_step(void *const *params, const void *const *grads,
     if (timed && (e = cudaEventRecord(ws->ev1, stream)) != cudaSuccess)
         return cuda_fail(e, "cudaEventRecord");
     st->grid = (int)(g2 * M);
-    if (stats_out) {
+    if (stats_out && norms_in) {
+        if (timed) {
+            if ((e = cudaEventSynchronize(ws->ev1)) != cudaSuccess)
+                return cuda_fail(e, "AdamW step");
+            float ms = -1.f;
+            if (cudaEventElapsedTime(&ms, ws->ev0, ws->ev1) == cudaSuccess)
+                st->kernel_ms = ms;
+            else
+                cudaGetLastError();
+        }
+    } else if (stats_out) {
         e = cudaMemcpyAsync(ws->host, a.out, 2 * ALOCO_MAX_WORKERS * sizeof(double),
                             cudaMemcpyDeviceToHost, stream);
         if (e == cudaSuccess) e = cudaStreamSynchronize(stream);

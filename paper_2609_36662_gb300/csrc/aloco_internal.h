@@ -159,6 +159,8 @@ struct AdamArgs {
     double max_norm;                    // clipping threshold; <= 0: none
     double *partials;                   // [M][g1] sums of g^2 (device)
     double *out;                        // [2][ALOCO_MAX_WORKERS]: norms, factors
+    int given;                          // 1: clip[] holds the factors; no norm pass
+    float clip[ALOCO_MAX_WORKERS];      // clipping factors when given
 };
 
 // Enqueue the norm pass (grid g1 x M) and the update pass (grid g2 x M).

@@ -324,3 +324,17 @@ def test_adamw_defaults_and_argument_errors(lib):
     assert "overlap" not in A.last_error()
     # N = 0 needs no device
     assert call(N=0) == A.OK
+    # given norms must be finite and non-negative
+    def normed(norms):
+        p = {k: [base + (4 * m + i) * MB for m in range(2)]
+             for i, k in enumerate(("x", "g", "m1", "m2"))}
+        arr = lambda v: (ctypes.c_void_p * 2)(*v)
+        nrm = (ctypes.c_double * 2)(*norms)
+        return lib.aloco_adamw_step_normed(arr(p["x"]), arr(p["g"]), arr(p["m1"]),
+                                           arr(p["m2"]), 1000, 2, A.F32, A.F32,
+                                           ctypes.byref(A.adamw_cfg()), nrm, None, None)
+    for bad in ([1.0, float("nan")], [-1.0, 2.0], [float("inf"), 1.0]):
+        assert normed(bad) == A.ERR_ARG and "grad_norms" in A.last_error()
+    assert lib.aloco_adamw_step_normed(None, None, None, None, 0, 1, A.F32, A.F32,
+                                       ctypes.byref(A.adamw_cfg()), None, None,
+                                       None) == A.ERR_ARG

@@ -199,3 +199,31 @@ def test_full_size_llama150m_eight_fp32_workers():
         assert_field(m2[m].cpu().numpy(), orc["m2"][0], f"v'[{m}]")
         assert st["grad_norm"][m] == pytest.approx(orc["norms"][0], rel=RTOL_STAT)
         del orc
+
+
+@pytest.mark.parametrize("pdt,gdt", [(O.F32, O.F32), (O.BF16, O.BF16), (O.BF16, O.F32)],
+                         ids=["p32g32", "p16g16", "p16g32"])
+def test_normed_step_equals_the_two_pass_step(pdt, gdt):
+    """Given the norms the two-pass step computed, the one-pass step forms
+    the same clipping factors and writes the same bits."""
+    N, M = 1_000_003, 5
+    a = _state(N, M, pdt, gdt, seed=77)
+    b = _state(N, M, pdt, gdt, seed=77)
+    cfg = A.adamw_cfg(**dict(C4, lr=4e-4, step=9))
+    st1 = A.adamw_step(*a, cfg)
+    st2 = A.adamw_step(*b, cfg, grad_norms=st1["grad_norm"])
+    assert st2["grad_norm"] == st1["grad_norm"]
+    assert st2["clip"] == st1["clip"] and min(st1["clip"]) < 1.0
+    for x, y in zip(sum(a[:1] + a[2:], []), sum(b[:1] + b[2:], [])):
+        bits = torch.int16 if x.dtype == torch.bfloat16 else torch.int32
+        assert torch.equal(x.view(bits), y.view(bits))
+
+
+def test_normed_step_matches_the_oracle():
+    """The oracle's norms in, the oracle's step out (fields within 1e-5)."""
+    N, M = 300_007, 3
+    xs, gs, m1, m2 = _state(N, M, O.F32, O.F32, seed=78)
+    cfg = dict(C4, lr=3e-4, step=5)
+    orc = _oracle(xs, gs, m1, m2, O.F32, O.F32, cfg)
+    st = A.adamw_step(xs, gs, m1, m2, A.adamw_cfg(**cfg), grad_norms=orc["norms"])
+    _compare(xs, m1, m2, st, orc, O.F32)
