@@ -84,7 +84,7 @@ def _load():
     lib.orc_adamw_step.restype = None
     lib.orc_adamw_step.argtypes = [vp, i32, vp, i32, vp, vp, i64, i32, dbl,
                                    dbl, dbl, dbl, dbl, dbl, i64, vp, vp, vp,
-                                   vp, dp]
+                                   vp, dp, vp]
     _lib = lib
     return lib
 
@@ -285,10 +285,11 @@ def int8_round(g, v, xs, dtype, parts, mu_t, eta_out, inv_norm, eps=1e-8):
 # ------------------------------------------------ inner AdamW step (Sec. 2)
 
 def adamw_step(xs, x_dtype, grads, g_dtype, m1s, m2s, lr, beta1, beta2, eps,
-               weight_decay, max_norm, step):
+               weight_decay, max_norm, step, norms=None):
     """One AdamW step (decoupled weight decay, per-replica gradient-norm
     clipping) on each replica.  xs / grads: float32 arrays, or bf16 bit
-    patterns (uint16) for dtype BF16; m1s, m2s: float32.  Returns the
+    patterns (uint16) for dtype BF16; m1s, m2s: float32.  norms (optional):
+    the gradients' norms over their whole replicas, for a slice.  Returns the
     unrounded float64 results, x' in its storage type and the pre-clipping
     gradient norms."""
     M = len(xs)
@@ -305,13 +306,15 @@ def adamw_step(xs, x_dtype, grads, g_dtype, m1s, m2s, lr, beta1, beta2, eps,
     m1_out = [np.empty(N, np.float64) for _ in range(M)]
     m2_out = [np.empty(N, np.float64) for _ in range(M)]
     x_store = [np.empty(N, xdt) for _ in range(M)]
-    norms = (ctypes.c_double * M)()
+    out_norms = (ctypes.c_double * M)()
+    given = None if norms is None else (ctypes.c_double * M)(*[float(x) for x in norms])
 
     def arr(lst):
         return (ctypes.c_void_p * M)(*[_ptr(a) for a in lst])
     _load().orc_adamw_step(arr(xs), x_dtype, arr(grads), g_dtype, arr(m1s),
                            arr(m2s), N, M, lr, beta1, beta2, eps,
                            weight_decay, max_norm, step, arr(x_out),
-                           arr(m1_out), arr(m2_out), arr(x_store), norms)
+                           arr(m1_out), arr(m2_out), arr(x_store), out_norms,
+                           given)
     return {"x": x_out, "m1": m1_out, "m2": m2_out, "x_store": x_store,
-            "norms": list(norms)}
+            "norms": list(out_norms)}

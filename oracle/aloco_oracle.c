@@ -427,23 +427,33 @@ int64_t orc_int8_round(const float *g, const float *v, const void *const *x,
  * applies to every parameter.  x and g may be fp32 or bf16 (widened
  * exactly); m, v are fp32.  Outputs are unrounded doubles, plus x' in its
  * storage type (fp32 rounding, or bf16 round-to-nearest-even) when x_store
- * is given; norms[m] = ||g_m|| before clipping. */
+ * is given; norms[m] = ||g_m|| before clipping.  With norms_in != NULL the
+ * norms are taken from it instead of the passed elements (for a slice of a
+ * longer replica). */
 void orc_adamw_step(const void *const *x, int x_dtype, const void *const *grad,
                     int g_dtype, const float *const *m1, const float *const *m2,
                     int64_t N, int M, double lr, double beta1, double beta2,
                     double eps, double weight_decay, double max_norm,
                     int64_t step, double *const *x_out, double *const *m1_out,
-                    double *const *m2_out, void *const *x_store, double *norms)
+                    double *const *m2_out, void *const *x_store, double *norms,
+                    const double *norms_in)
 {
     double bc1 = 1.0 - pow(beta1, (double)step);
     double bc2 = 1.0 - pow(beta2, (double)step);
     for (int m = 0; m < M; ++m) {
-        double ss = 0.0;
-        for (int64_t i = 0; i < N; ++i) {
-            double g = orc_replica(grad[m], g_dtype, i);
-            ss += g * g;
+        double norm;
+        if (norms_in) {
+            /* the gradient's norm over its whole replica, supplied when only a
+             * slice of the replica is passed */
+            norm = norms_in[m];
+        } else {
+            double ss = 0.0;
+            for (int64_t i = 0; i < N; ++i) {
+                double g = orc_replica(grad[m], g_dtype, i);
+                ss += g * g;
+            }
+            norm = sqrt(ss);
         }
-        double norm = sqrt(ss);
         norms[m] = norm;
         double c = 1.0;
         if (max_norm > 0.0) {

@@ -155,3 +155,20 @@ def test_bf16_inputs_are_widened_and_the_result_rounded_to_nearest_even():
     np.testing.assert_array_equal(orc["x"][0], ref["x"][0])
     want = torch.from_numpy(ref["x"][0]).to(torch.bfloat16)
     np.testing.assert_array_equal(orc["x_store"][0], bits(want))
+
+
+def test_given_norms_reproduce_the_whole_replica_step_on_a_slice():
+    """A slice stepped with the whole replica's norm equals that slice of
+    the whole step (the clipping factor is the only coupling)."""
+    rng = np.random.default_rng(8)
+    n = 5000
+    x, g = _f32(rng, n, 0.02), _f32(rng, n, 0.1)
+    m1, m2 = _f32(rng, n, 1e-3), np.abs(_f32(rng, n, 1e-4))
+    whole = O.adamw_step([x], O.F32, [g], O.F32, [m1], [m2], 1e-3, step=6, **C4)
+    sl = slice(1234, 3456)
+    part = O.adamw_step([x[sl]], O.F32, [g[sl]], O.F32, [m1[sl]], [m2[sl]], 1e-3,
+                        step=6, norms=whole["norms"], **C4)
+    assert whole["norms"][0] > 1.0            # clipping active
+    for k in ("x", "m1", "m2"):
+        np.testing.assert_array_equal(part[k][0], whole[k][0][sl])
+    assert part["norms"] == whole["norms"]
