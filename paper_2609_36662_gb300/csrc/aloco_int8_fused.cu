@@ -3,12 +3,14 @@
 //
 // CTAs of T threads work through 4096-element codec blocks (grid stride),
 // 4096 / T consecutive elements per thread: one 1024-thread CTA per SM, or
-// two 512-thread CTAs per SM (bf16 with M >= 5; see fused_threads).  Per
+// two 512-thread CTAs per SM (bf16 except M = 2; see fused_threads).  Per
 // block:
 //   1. theta, v and the M replica slices are staged in shared memory with
 //      cp.async; each thread copies exactly the 16- or 8-byte chunks it later
-//      reads, so the staging needs no barrier.  With two staging buffers the
-//      next block's copies are issued before this block is computed;
+//      reads, so the staging needs no barrier, and one buffer serves: the
+//      next block's copies are issued as soon as the thread has read its own
+//      chunks of this block (before the mean's codec, the outer step and the
+//      stores), so they overlap the rest of the block;
 //   2. each warp reduces every worker's max |Delta_m| (as float bits, NaN
 //      above +inf); barrier; every warp then reads the 32 warp maxima of each
 //      worker lane-parallel and folds them with one warp max, and lane m
@@ -23,10 +25,11 @@
 // arithmetic of every element is the split form's (aloco_int8.cu), so both
 // forms give the same codes, scales and outputs.
 //
-// Shared memory per staging buffer: 4096 x (8 + M x element size) bytes.
-// The 1024-thread shape takes two buffers where they fit in 200 KB (fp32
-// M <= 4, bf16 M <= 4), else one; the 512-thread shape one per CTA.  Worker
-// counts beyond 8 use the split form.
+// Shared memory per CTA: one staging buffer of 4096 x (8 + M x element
+// size) bytes (bf16 with 1024 threads and odd M: one more worker's slot).
+// A second buffer, issuing the next block's copies before this block is
+// computed, measured no faster anywhere and halves the room for the 512-
+// thread shape.  Worker counts beyond 8 use the split form.
 #include <atomic>
 
 #include "aloco_int8.cuh"
@@ -39,12 +42,12 @@ constexpr int kFlushBlocks = 8;
 constexpr int kFusedMax = 8;
 
 // Threads per CTA (T) and elements per thread (4096 / T), measured on
-// GB300 over M = 1..8 and both replica types (2^26-parameter rounds,
-// fraction of the copy peak):
-//   T = 1024, one CTA per SM, double-buffered staging: fp32 0.76-0.84
-//     (M <= 4) and 0.66-0.71 (M = 5..8), bf16 0.64-0.66 (M <= 4);
-//   T = 512, two CTAs per SM, one buffer each: bf16 0.62-0.65 for M = 5..8,
-//     against 0.54-0.62 with 1024 threads.
+// GB300 (2^26-parameter rounds, fraction of the measured copy peak):
+//   fp32: T = 1024 (one CTA per SM) 0.78-0.87 over M = 1..8; T = 512 (two
+//     CTAs per SM) 0.58-0.72;
+//   bf16: T = 512 0.65-0.71 over M = 1, 3..8 against 0.60-0.67 with 1024
+//     threads; at M = 2, where the 1024-thread shape's worker pair fills one
+//     16-byte slot, 1024 threads 0.69 against 0.65.
 // ALOCO_I8_FUSED_T = 512 or 1024 forces one shape (a tuning knob).
 #ifndef ALOCO_I8_FUSED_T
 #define ALOCO_I8_FUSED_T 0
@@ -52,7 +55,7 @@ constexpr int kFusedMax = 8;
 template <int M, bool BF16>
 constexpr int fused_threads() {
     if (ALOCO_I8_FUSED_T) return ALOCO_I8_FUSED_T;
-    return (BF16 && M >= 5) ? 512 : 1024;
+    return (BF16 && M != 2) ? 512 : 1024;
 }
 
 // Replica staging of a thread's PER elements: fp32 workers one after
@@ -68,12 +71,6 @@ __host__ __device__ constexpr size_t rep_bytes() {
 template <int M, bool BF16, int T>
 __host__ __device__ constexpr size_t stage_bytes() {
     return (size_t)kI8Block * 8 + rep_bytes<M, BF16, T>();
-}
-// Two staging buffers where they fit one 1024-thread CTA per SM; the
-// 512-thread shape runs two CTAs per SM with one buffer each.
-template <int M, bool BF16, int T>
-__host__ __device__ constexpr int n_bufs() {
-    return (T == 1024 && 2 * stage_bytes<M, BF16, T>() <= 200 * 1024) ? 2 : 1;
 }
 template <int T>
 __host__ __device__ constexpr int fused_min_ctas() { return T == 512 ? 2 : 1; }
@@ -228,8 +225,6 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
     constexpr int PER = kI8Block / T;  // elements per thread
     constexpr int NP = PER / 2;        // pairs per thread
     constexpr int W = T / 32;          // warps
-    constexpr int NB = n_bufs<M, BF16, T>();
-    constexpr size_t SB = stage_bytes<M, BF16, T>();
     // Single buffers suffice: red_w is read between the block's two
     // barriers and rewritten only after the second; red1 is read after the
     // second and rewritten only after the next block's first.
@@ -274,7 +269,6 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
                                 len == kI8Block && a.nvec > 0 && (start % 8) == 0, t);
         cp_commit();
     }
-    int buf = 0;
     for (; kb < nblocks; kb += gridDim.x) {
         const bool full = len == kI8Block;
         const bool vec = a.nvec > 0 && (start % 8) == 0;
@@ -282,17 +276,8 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
         int64_t nstart = 0;
         int nlen = 0;
         if (nk < nblocks) locate_block(P, nk, nstart, nlen);
-        if constexpr (NB == 2) {
-            if (nk < nblocks)
-                stage_block<M, BF16, T>(stage + (buf ^ 1) * SB, a, nstart, nlen,
-                                        nlen == kI8Block && a.nvec > 0 && (nstart % 8) == 0, t);
-            cp_commit();
-            cp_wait<1>();  // all but the group just issued: this block's copies
-        } else {
-            cp_wait<0>();
-        }
-        const unsigned char *sb = stage + buf * SB;
-        const float *sg = reinterpret_cast<const float *>(sb);
+        cp_wait<0>();  // this thread's copies of this block
+        const float *sg = reinterpret_cast<const float *>(stage);
         const float *sv = sg + kI8Block;
         const unsigned char *sx = reinterpret_cast<const unsigned char *>(sv + kI8Block);
 
@@ -392,6 +377,19 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
         }
 
         // 4. the mean's codec, the outer step and the stores
+        float v[PER];
+#pragma unroll
+        for (int c = 0; c < PER; c += 4) {
+            const float4 q = *reinterpret_cast<const float4 *>(sv + e0 + c);
+            v[c] = q.x; v[c + 1] = q.y; v[c + 2] = q.z; v[c + 3] = q.w;
+        }
+        // this thread has read all of its staged chunks: their slots take
+        // the next block's copies while the rest of this block runs
+        if (nk < nblocks) {
+            stage_block<M, BF16, T>(stage, a, nstart, nlen,
+                                    nlen == kI8Block && a.nvec > 0 && (nstart % 8) == 0, t);
+            cp_commit();
+        }
         float sum[PER];
 #pragma unroll
         for (int j = 0; j < NP; ++j) {
@@ -404,12 +402,6 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
         // elements beyond a short block hold 0 and do not move the maximum
         const float s = codec_scale(block_amax<PER, W>(sum, red1));
         const float rs = __frcp_rn(s);
-        float v[PER];
-#pragma unroll
-        for (int c = 0; c < PER; c += 4) {
-            const float4 q = *reinterpret_cast<const float4 *>(sv + e0 + c);
-            v[c] = q.x; v[c + 1] = q.y; v[c + 2] = q.z; v[c + 3] = q.w;
-        }
         float gp[PER], vp[PER];
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
@@ -467,15 +459,6 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
         b64 += (double)b32;  // at most PER terms per thread and block
         b32 = 0.f;
 
-        if constexpr (NB == 1) {
-            if (nk < nblocks) {
-                stage_block<M, BF16, T>(stage, a, nstart, nlen,
-                                        nlen == kI8Block && a.nvec > 0 && (nstart % 8) == 0, t);
-                cp_commit();
-            }
-        } else {
-            buf ^= 1;
-        }
         start = nstart;
         len = nlen;
     }
@@ -501,7 +484,7 @@ template <int M, bool BF16>
 cudaError_t fused_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
                          int max_grid, cudaStream_t stream, int *grid_out) {
     constexpr int T = fused_threads<M, BF16>();
-    constexpr size_t smem = n_bufs<M, BF16, T>() * stage_bytes<M, BF16, T>();
+    constexpr size_t smem = stage_bytes<M, BF16, T>();
     static PerDevice occ_cache;  // attribute set-up and occupancy, per device
     const int dev = PerDevice::device();
     int occ = occ_cache.get(dev);
