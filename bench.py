@@ -83,11 +83,11 @@ def hbm_peak():
 KERNEL_SOURCES = {
     "sync_kernel": ("aloco_sync_kernel.cuh", "aloco_sync_f32.cu",
                     "aloco_sync_bf16.cu"),
-    "sync_tma_kernel": ("aloco_sync_kernel.cuh", "aloco_sync_tma.cuh",
+    "sync_tma_kernel": ("aloco_sync_kernel.cuh", "aloco_bulk.cuh", "aloco_sync_tma.cuh",
                         "aloco_sync_tma_f32.cu", "aloco_sync_tma_bf16.cu"),
     "int8_split_kernels": ("aloco_sync_kernel.cuh", "aloco_int8.cuh",
                            "aloco_int8.cu"),
-    "int8_fused_kernel": ("aloco_sync_kernel.cuh", "aloco_int8.cuh",
+    "int8_fused_kernel": ("aloco_sync_kernel.cuh", "aloco_bulk.cuh", "aloco_int8.cuh",
                           "aloco_int8_fused.cu"),
     "adamw_kernels": ("aloco_sync_kernel.cuh", "aloco_adamw.cu"),
 }

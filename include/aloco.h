@@ -604,13 +604,14 @@ int aloco_sync_noalloc(float *global, float *momentum, void *const *locals,
                        aloco_stats_t *stats_out);
 
 /* TESTING ONLY (failure detection without a GPU fault): the calling
- * thread's next aloco_sync / aloco_sync_ex round that runs the bulk-copy
- * pass skips the copies of tile `tile` (a negative value cancels).  That
- * stage's mbarrier then never completes, so its consumers' bounded wait
- * (about 2 s) runs out: the block aborts, lets its copies in flight land,
- * and the round returns ALOCO_ERR_CUDA with every kernel finished and the
- * device usable.  The hook is consumed by that round; no other call reads
- * it. */
+ * thread's next round that runs the bulk-copy pass (aloco_sync /
+ * aloco_sync_ex) or the fused INT8 pass (aloco_sync_int8) skips the copies
+ * of tile `tile` (bulk-copy pass) or of codec block `tile` (fused INT8
+ * pass, a whole aligned block); a negative value cancels.  That stage's
+ * mbarrier then never completes, so the bounded waits on it (about 2 s) run
+ * out: the block aborts, lets its copies in flight land, and the round
+ * returns ALOCO_ERR_CUDA with every kernel finished and the device usable.
+ * The hook is consumed by that round; no other call reads it. */
 void aloco_test_stall_tile(int64_t tile);
 
 /* Message of the last failure on the calling thread ("" if none).  The

@@ -277,7 +277,7 @@ GetAddressRangeFn address_range_fn() {
 // Helpers with external linkage: also used by the allocation-free entry
 // point (aloco_noalloc.cu).
 // Testing hook of aloco_test_stall_tile: consumed by the calling thread's
-// next bulk-copy round.
+// next bulk-copy or fused INT8 round.
 thread_local int64_t t_test_stall_tile1 = 0;
 
 namespace aloco {
@@ -583,7 +583,7 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     a.n_tiles = plan.tiles;
     a.stages = plan.stages;
     a.error = ws->error;
-    if (tma) {
+    if (tma || fused) {
         a.test_stall_tile1 = t_test_stall_tile1;
         t_test_stall_tile1 = 0;
     }

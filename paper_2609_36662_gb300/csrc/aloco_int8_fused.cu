@@ -2,36 +2,46 @@
 // read from HBM once, as in the uncompressed round.
 //
 // CTAs of T threads work through 4096-element codec blocks (grid stride),
-// 4096 / T consecutive elements per thread: one 1024-thread CTA per SM, or
-// two 512-thread CTAs per SM (bf16 except M = 2; see fused_threads).  Per
-// block:
-//   1. theta, v and the M replica slices are staged in shared memory with
-//      cp.async; each thread copies exactly the 16- or 8-byte chunks it later
-//      reads, so the staging needs no barrier, and one buffer serves: the
-//      next block's copies are issued as soon as the thread has read its own
-//      chunks of this block (before the mean's codec, the outer step and the
-//      stores), so they overlap the rest of the block;
+// 4096 / T elements per thread in chunks of 4 (chunk c of thread t at
+// 4t + c x 4T, so warp accesses to shared memory are contiguous): two
+// 512-thread CTAs per SM where they fit, else one 1024-thread CTA (see
+// fused_threads).  Per block:
+//   1. theta, v and the M replica slices arrive in shared memory by bulk
+//      copies (cp.async.bulk, one per array, issued by thread 0 and
+//      completing on the CTA's mbarrier; every thread's wait on it is
+//      bounded).  Short or unaligned blocks (tensor ends) are instead staged
+//      by every thread, element by element, into its own slots;
 //   2. each warp reduces every worker's max |Delta_m| (as float bits, NaN
-//      above +inf); barrier; every warp then reads the 32 warp maxima of each
-//      worker lane-parallel and folds them with one warp max, and lane m
-//      turns worker m's maximum into its scale and reciprocal;
+//      above +inf); barrier 1; every warp then reads the 32 warp maxima of
+//      each worker lane-parallel and folds them with one warp max, and lane
+//      m turns worker m's maximum into its scale and reciprocal;
 //   3. the workers' pseudo-gradients are encoded, decoded and summed in FP32
 //      worker order, reading the replicas again from shared memory;
-//   4. the mean is encoded and decoded once (its block maximum is the second
-//      barrier), the corrected Nesterov step runs, and theta', v' and the
-//      reset replicas are stored.
+//   4. the mean is encoded and decoded once (its block maximum is barrier 2).
+//      Every thread has then read this block's staging, so thread 0 issues
+//      the next block's bulk copies into the same buffer; they overlap the
+//      outer step and the stores;
+//   5. theta' is written once, in the replica type, to an output tile in
+//      shared memory (theta' and v' in fp32 too where they fit), and after
+//      the next block's barrier 1 thread 0 stores the tiles with bulk
+//      copies: the M replica resets are M copies of one tile.  Before
+//      barrier 2 of that block it waits until they have read the tiles.
 // Drift energies sum in fp32 per thread over at most 8 blocks (32 squares)
 // before each warp adds them, in a fixed order, to its fp64 row.  The
 // arithmetic of every element is the split form's (aloco_int8.cu), so both
 // forms give the same codes, scales and outputs.
 //
-// Shared memory per CTA: one staging buffer of 4096 x (8 + M x element
-// size) bytes (bf16 with 1024 threads and odd M: one more worker's slot).
-// A second buffer, issuing the next block's copies before this block is
-// computed, measured no faster anywhere and halves the room for the 512-
-// thread shape.  Worker counts beyond 8 use the split form.
+// Shared memory per CTA: the input buffer, 4096 x (8 + M x element size)
+// bytes, and the output tiles, 4096 x element size (plus 4096 x 8 for the
+// fp32 theta' and v' tiles where they fit; elsewhere threads store theta'
+// and v' themselves).  Worker counts beyond 8 use the split form.
+//
+// A bounded wait that runs out (about 2 s) sets the round's error word; the
+// whole CTA leaves the block loop together at the next barrier, thread 0
+// lets the copies it issued land, and the host reports the error.
 #include <atomic>
 
+#include "aloco_bulk.cuh"
 #include "aloco_int8.cuh"
 
 namespace aloco {
@@ -41,161 +51,100 @@ namespace {
 constexpr int kFlushBlocks = 8;
 constexpr int kFusedMax = 8;
 
+// Shared memory of one SM and the largest a CTA may take (bytes), and the
+// part of each CTA's share the system reserves.
+constexpr size_t kSmemPerSm = 233472;
+constexpr size_t kSmemPerCta = 232448;
+constexpr size_t kSmemReserved = 1024;
+
+template <bool BF16>
+__host__ __device__ constexpr int esize() { return BF16 ? 2 : 4; }
+// theta, v (fp32) and the M replica slices of one block
+template <int M, bool BF16>
+__host__ __device__ constexpr size_t in_bytes() {
+    return (size_t)kI8Block * (8 + M * esize<BF16>());
+}
+// the static shared arrays of the kernel and of the final reduction (an
+// upper bound)
+template <int M, int T>
+__host__ __device__ constexpr size_t static_bytes() {
+    return (size_t)(T / 32) * (4 * M + 4 + 8 * M + 8 * (M + 1)) + 4096;
+}
+template <int T>
+__host__ __device__ constexpr size_t cta_budget() {
+    return T == 512 ? kSmemPerSm / 2 - kSmemReserved : kSmemPerCta;
+}
+// The fp32 theta' and v' tiles fit beside the input and the replica tile.
+template <int M, bool BF16, int T>
+__host__ __device__ constexpr bool tile_gv() {
+    return in_bytes<M, BF16>() + (size_t)kI8Block * (esize<BF16>() + (BF16 ? 8 : 4)) +
+               static_bytes<M, T>() <=
+           cta_budget<T>();
+}
+template <int M, bool BF16, int T>
+__host__ __device__ constexpr size_t out_bytes() {
+    return tile_gv<M, BF16, T>() ? (size_t)kI8Block * (esize<BF16>() + (BF16 ? 8 : 4))
+                                 : (size_t)kI8Block * esize<BF16>();
+}
+template <int M, bool BF16, int T>
+__host__ __device__ constexpr size_t fused_smem() {
+    return in_bytes<M, BF16>() + out_bytes<M, BF16, T>();
+}
+template <int M, bool BF16, int T>
+__host__ __device__ constexpr bool fits() {
+    return fused_smem<M, BF16, T>() + static_bytes<M, T>() <= cta_budget<T>();
+}
+
 // Threads per CTA (T) and elements per thread (4096 / T), measured on
 // GB300 (2^26-parameter rounds, fraction of the measured copy peak):
-//   fp32: T = 1024 (one CTA per SM) 0.78-0.87 over M = 1..8; T = 512 (two
-//     CTAs per SM) 0.58-0.72;
-//   bf16: T = 512 0.65-0.71 over M = 1, 3..8 against 0.60-0.67 with 1024
-//     threads; at M = 2, where the 1024-thread shape's worker pair fills one
-//     16-byte slot, 1024 threads 0.69 against 0.65.
+//   bf16: T = 512, two CTAs per SM, 0.85 for M <= 4 and 0.77-0.79 for
+//     M = 6, 8, against 0.63-0.67 with one 1024-thread CTA, whose single
+//     block in flight leaves the SM idle while the next block's copies land;
+//   fp32: T = 512 0.88-0.93 for M <= 3, against 0.70-0.82 with 1024
+//     threads; from M = 4 two 512-thread CTAs no longer fit.
 // ALOCO_I8_FUSED_T = 512 or 1024 forces one shape (a tuning knob).
 #ifndef ALOCO_I8_FUSED_T
 #define ALOCO_I8_FUSED_T 0
 #endif
 template <int M, bool BF16>
 constexpr int fused_threads() {
-    if (ALOCO_I8_FUSED_T) return ALOCO_I8_FUSED_T;
-    return (BF16 && M != 2) ? 512 : 1024;
-}
-
-// Replica staging of a thread's PER elements: fp32 workers one after
-// another (16 KB each).  bf16 at 4 elements per thread: workers in pairs, a
-// thread's elements of workers 2p and 2p + 1 side by side in one 16-byte
-// slot, so one shared-memory load feeds both; at 8 elements per thread each
-// worker's slice is already one 16-byte load, one worker after another.
-template <int M, bool BF16, int T>
-__host__ __device__ constexpr size_t rep_bytes() {
-    return (BF16 && T == 1024) ? (size_t)((M + 1) / 2) * kI8Block * 4
-                               : (size_t)M * kI8Block * (BF16 ? 2 : 4);
-}
-template <int M, bool BF16, int T>
-__host__ __device__ constexpr size_t stage_bytes() {
-    return (size_t)kI8Block * 8 + rep_bytes<M, BF16, T>();
+    constexpr int want = ALOCO_I8_FUSED_T ? ALOCO_I8_FUSED_T : 512;
+    return (want == 512 && !fits<M, BF16, 512>()) ? 1024 : want;
 }
 template <int T>
 __host__ __device__ constexpr int fused_min_ctas() { return T == 512 ? 2 : 1; }
-// Byte offset of worker m's element e (of 4096) in the replica staging.
-template <bool BF16, int T>
-__device__ __forceinline__ int rep_off(int m, int e) {
-    if constexpr (BF16 && T == 1024)
-        return ((m >> 1) * T + (e >> 2)) * 16 + (m & 1) * 8 + (e & 3) * 2;
-    else
-        return m * kI8Block * (BF16 ? 2 : 4) + e * (BF16 ? 2 : 4);
-}
-
-__device__ __forceinline__ void cp16(void *smem, const void *gmem) {
-    const unsigned d = (unsigned)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gmem)
-                 : "memory");
-}
-__device__ __forceinline__ void cp8(void *smem, const void *gmem) {
-    const unsigned d = (unsigned)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(d), "l"(gmem)
-                 : "memory");
-}
-__device__ __forceinline__ void cp_commit() {
-    asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-// Stage one block: theta, v, then the replicas; thread t copies elements
-// [PER t, PER t + PER) of every array (16-byte copies; 8-byte for bf16 at 4
-// elements per thread).  Short or unaligned blocks are loaded element by
-// element, zero beyond the end.
-template <int M, bool BF16, int T>
-__device__ __forceinline__ void stage_block(unsigned char *buf, const SyncArgs &a,
-                                            int64_t start, int len, bool fast, int t) {
-    constexpr int PER = kI8Block / T;
-    float *sg = reinterpret_cast<float *>(buf);
-    float *sv = sg + kI8Block;
-    unsigned char *sx = reinterpret_cast<unsigned char *>(sv + kI8Block);
-    const int e = PER * t;
-    if (fast) {
-#pragma unroll
-        for (int c = 0; c < PER; c += 4) {
-            cp16(sg + e + c, a.g + start + e + c);
-            cp16(sv + e + c, a.v + start + e + c);
-        }
-#pragma unroll
-        for (int m = 0; m < M; ++m) {
-            if constexpr (BF16) {
-                const uint16_t *src = reinterpret_cast<const uint16_t *>(a.x[m]) + start + e;
-                if constexpr (PER == 4)
-                    cp8(sx + rep_off<true, T>(m, e), src);
-                else
-                    cp16(sx + rep_off<true, T>(m, e), src);
-            } else {
-#pragma unroll
-                for (int c = 0; c < PER; c += 4)
-                    cp16(sx + rep_off<false, T>(m, e + c),
-                         reinterpret_cast<const float *>(a.x[m]) + start + e + c);
-            }
-        }
-    } else {
-#pragma unroll
-        for (int k = 0; k < PER; ++k) {
-            const bool in = e + k < len;
-            sg[e + k] = in ? a.g[start + e + k] : 0.f;
-            sv[e + k] = in ? a.v[start + e + k] : 0.f;
-#pragma unroll
-            for (int m = 0; m < M; ++m) {
-                if constexpr (BF16)
-                    *reinterpret_cast<uint16_t *>(sx + rep_off<true, T>(m, e + k)) =
-                        in ? reinterpret_cast<const uint16_t *>(a.x[m])[start + e + k]
-                           : (uint16_t)0;
-                else
-                    *reinterpret_cast<float *>(sx + rep_off<false, T>(m, e + k)) =
-                        in ? reinterpret_cast<const float *>(a.x[m])[start + e + k] : 0.f;
-            }
-        }
-    }
-}
-
-__device__ __forceinline__ void widen4(uint32_t w0, uint32_t w1, float2 *o) {
-    o[0] = make_float2(bf16_lo(w0), bf16_hi(w0));
-    o[1] = make_float2(bf16_lo(w1), bf16_hi(w1));
-}
 
 // A thread's replica values of workers m0 and m0 + 1 (when m0 + 1 < M),
-// widened exactly, as PER / 2 pairs each.
+// widened exactly, as PER / 2 pairs each.  Worker m's slice starts at
+// m x 4096 x element size; thread t's chunks of 4 elements sit at 4t + c x 4T.
 template <int M, bool BF16, int T>
 __device__ __forceinline__ void staged_reps(const unsigned char *sx, int m0, int t,
                                             float2 (&a)[kI8Block / T / 2],
                                             float2 (&b)[kI8Block / T / 2]) {
     constexpr int PER = kI8Block / T;
-    const int e = PER * t;
-    if constexpr (BF16 && PER == 4) {
-        if (m0 + 1 < M) {
-            const uint4 w = *reinterpret_cast<const uint4 *>(sx + rep_off<true, T>(m0, e));
-            widen4(w.x, w.y, a);
-            widen4(w.z, w.w, b);
-        } else {
-            const uint2 w = *reinterpret_cast<const uint2 *>(sx + rep_off<true, T>(m0, e));
-            widen4(w.x, w.y, a);
-        }
-    } else if constexpr (BF16) {
-        const uint4 w = *reinterpret_cast<const uint4 *>(sx + rep_off<true, T>(m0, e));
-        widen4(w.x, w.y, a);
-        widen4(w.z, w.w, a + 2);
-        if (m0 + 1 < M) {
-            const uint4 u = *reinterpret_cast<const uint4 *>(sx + rep_off<true, T>(m0 + 1, e));
-            widen4(u.x, u.y, b);
-            widen4(u.z, u.w, b + 2);
-        }
-    } else {
+    constexpr int ES = esize<BF16>();
+    const unsigned char *p0 = sx + (size_t)m0 * kI8Block * ES + 4 * t * ES;
+    const unsigned char *p1 = p0 + kI8Block * ES;
 #pragma unroll
-        for (int c = 0; c < PER; c += 4) {
-            const float4 q = *reinterpret_cast<const float4 *>(sx + rep_off<false, T>(m0, e + c));
-            a[c / 2] = make_float2(q.x, q.y);
-            a[c / 2 + 1] = make_float2(q.z, q.w);
+    for (int c = 0; c < PER / 4; ++c) {
+        const int off = c * 4 * T * ES;
+        if constexpr (BF16) {
+            const uint2 w = *reinterpret_cast<const uint2 *>(p0 + off);
+            a[2 * c] = make_float2(bf16_lo(w.x), bf16_hi(w.x));
+            a[2 * c + 1] = make_float2(bf16_lo(w.y), bf16_hi(w.y));
             if (m0 + 1 < M) {
-                const float4 r =
-                    *reinterpret_cast<const float4 *>(sx + rep_off<false, T>(m0 + 1, e + c));
-                b[c / 2] = make_float2(r.x, r.y);
-                b[c / 2 + 1] = make_float2(r.z, r.w);
+                const uint2 u = *reinterpret_cast<const uint2 *>(p1 + off);
+                b[2 * c] = make_float2(bf16_lo(u.x), bf16_hi(u.x));
+                b[2 * c + 1] = make_float2(bf16_lo(u.y), bf16_hi(u.y));
+            }
+        } else {
+            const float4 q = *reinterpret_cast<const float4 *>(p0 + off);
+            a[2 * c] = make_float2(q.x, q.y);
+            a[2 * c + 1] = make_float2(q.z, q.w);
+            if (m0 + 1 < M) {
+                const float4 r = *reinterpret_cast<const float4 *>(p1 + off);
+                b[2 * c] = make_float2(r.x, r.y);
+                b[2 * c + 1] = make_float2(r.z, r.w);
             }
         }
     }
@@ -225,6 +174,10 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
     constexpr int PER = kI8Block / T;  // elements per thread
     constexpr int NP = PER / 2;        // pairs per thread
     constexpr int W = T / 32;          // warps
+    constexpr int ES = esize<BF16>();
+    constexpr bool GV = tile_gv<M, BF16, T>();
+    constexpr uint32_t kGVBytes = kI8Block * 4;  // one fp32 array of a block
+    constexpr uint32_t kXBytes = kI8Block * ES;  // one replica slice
     // Single buffers suffice: red_w is read between the block's two
     // barriers and rewritten only after the second; red1 is read after the
     // second and rewritten only after the next block's first.
@@ -232,11 +185,24 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
     __shared__ unsigned red1[W];
     __shared__ double e_w[W][M];
     __shared__ __align__(16) float2 sr[W][M + (M & 1)];  // per warp: (scale, 1/scale)
-    extern __shared__ __align__(16) unsigned char stage[];
+    __shared__ __align__(8) unsigned long long full_bar;
+    extern __shared__ __align__(128) unsigned char smem[];
+    float *sg = reinterpret_cast<float *>(smem);
+    float *sv = sg + kI8Block;
+    unsigned char *sx = smem + 2 * kGVBytes;
+    unsigned char *ox = sx + M * kXBytes;             // theta' in the replica type
+    float *og = BF16 ? reinterpret_cast<float *>(ox + kXBytes)  // theta' (fp32)
+                     : reinterpret_cast<float *>(ox);
+    float *ov = og + kI8Block;                         // v' (GV only)
+    const uint32_t bar = smem_addr(&full_bar);
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     if (lane < M) e_w[warp][lane] = 0.0;
-    __syncwarp();
+    if (t == 0) {
+        mbar_init(bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
     float e_acc[M];
 #pragma unroll
     for (int m = 0; m < M; ++m) e_acc[m] = 0.f;
@@ -258,33 +224,96 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
     unsigned nf = 0;
     const Coef k{a.c_hi, a.c_lo, a.mu_hi, a.mu_lo, a.neg_eta_hi, a.neg_eta_lo};
     const int64_t nblocks = P.blk[P.n_parts];
-    const int e0 = PER * t;
+    // thread t holds the 4-element chunks at 4t + c x 4T (c < PER / 4), so
+    // every warp access to a staged array is contiguous
+    auto el = [&](int i) { return (i >> 2) * (4 * T) + 4 * t + (i & 3); };
+
+    // whole blocks at 16-byte aligned addresses move by bulk copies
+    auto bulk_block = [&](int64_t s, int l) {
+        return l == kI8Block && a.nvec > 0 && (s % 8) == 0;
+    };
+    bool in_flight = false;  // thread 0: bulk loads issued and not yet seen complete
+    // thread 0: the bulk copies of the block at s
+    auto stage_bulk = [&](int64_t kbi, int64_t s) {
+        if (a.test_stall_tile1 != 0 && kbi == a.test_stall_tile1 - 1)
+            return;  // testing only: this phase never completes
+        mbar_arrive_expect_tx(bar, 2 * kGVBytes + M * kXBytes);
+        bulk_load(smem_addr(sg), a.g + s, kGVBytes, bar);
+        bulk_load(smem_addr(sv), a.v + s, kGVBytes, bar);
+#pragma unroll
+        for (int m = 0; m < M; ++m)
+            bulk_load(smem_addr(sx + m * kXBytes),
+                      reinterpret_cast<const unsigned char *>(a.x[m]) + s * ES, kXBytes, bar);
+        in_flight = true;
+    };
+    // every thread: its own elements of a short or unaligned block
+    auto stage_own = [&](int64_t s, int l) {
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int e = el(i);
+            const bool in = e < l;
+            sg[e] = in ? a.g[s + e] : 0.f;
+            sv[e] = in ? a.v[s + e] : 0.f;
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                if constexpr (BF16)
+                    reinterpret_cast<uint16_t *>(sx + m * kXBytes)[e] =
+                        in ? reinterpret_cast<const uint16_t *>(a.x[m])[s + e]
+                           : (uint16_t)0;
+                else
+                    reinterpret_cast<float *>(sx + m * kXBytes)[e] =
+                        in ? reinterpret_cast<const float *>(a.x[m])[s + e] : 0.f;
+            }
+        }
+        // a later bulk copy may overwrite these bytes
+        fence_proxy_async_smem();
+    };
+    // thread 0: the output tiles of the block at s go to global memory
+    auto store_tiles = [&](int64_t s) {
+        if constexpr (GV) {
+            bulk_store(a.g + s, smem_addr(og), kGVBytes);
+            bulk_store(a.v + s, smem_addr(ov), kGVBytes);
+        }
+#pragma unroll
+        for (int m = 0; m < M; ++m)
+            bulk_store(reinterpret_cast<unsigned char *>(a.x[m]) + s * ES, smem_addr(ox),
+                       kXBytes);
+        bulk_commit();
+    };
 
     int64_t kb = blockIdx.x;
     int64_t start = 0;
     int len = 0;
+    uint32_t phase = 0;
+    bool pend = false;  // the previous block's tiles wait for their bulk stores
+    int64_t pstart = 0;
+    bool failed = false;
     if (kb < nblocks) {
         locate_block(P, kb, start, len);
-        stage_block<M, BF16, T>(stage, a, start, len,
-                                len == kI8Block && a.nvec > 0 && (start % 8) == 0, t);
-        cp_commit();
+        if (!bulk_block(start, len))
+            stage_own(start, len);
+        else if (t == 0)
+            stage_bulk(kb, start);
     }
     for (; kb < nblocks; kb += gridDim.x) {
         const bool full = len == kI8Block;
-        const bool vec = a.nvec > 0 && (start % 8) == 0;
+        const bool bulk = bulk_block(start, len);
         const int64_t nk = kb + gridDim.x;
         int64_t nstart = 0;
         int nlen = 0;
         if (nk < nblocks) locate_block(P, nk, nstart, nlen);
-        cp_wait<0>();  // this thread's copies of this block
-        const float *sg = reinterpret_cast<const float *>(stage);
-        const float *sv = sg + kI8Block;
-        const unsigned char *sx = reinterpret_cast<const unsigned char *>(sv + kI8Block);
+        const bool next_bulk = nk < nblocks && bulk_block(nstart, nlen);
+        bool timed_out = false;
+        if (bulk) {
+            timed_out = !mbar_wait(bar, phase, nullptr);
+            if (t == 0 && !timed_out) in_flight = false;
+            phase ^= 1;
+        }
 
         float g[PER];
 #pragma unroll
         for (int c = 0; c < PER; c += 4) {
-            const float4 q = *reinterpret_cast<const float4 *>(sg + e0 + c);
+            const float4 q = *reinterpret_cast<const float4 *>(sg + el(c));
             g[c] = q.x; g[c + 1] = q.y; g[c + 2] = q.z; g[c + 3] = q.w;
         }
         float2 g2[NP];
@@ -324,7 +353,15 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
             if (m + 1 < M) worker_max(m + 1, xb);
         }
         if (++since_flush == kFlushBlocks) flush();
-        __syncthreads();
+        // barrier 1; a wait that ran out in any thread stops the whole CTA
+        if (__syncthreads_or(timed_out)) {
+            failed = true;
+            break;
+        }
+        // every thread wrote its part of the previous block's tiles before
+        // the barrier
+        if (pend && t == 0) store_tiles(pstart);
+        pend = false;
         {
             // every warp folds the W warp maxima of each worker (lane w reads
             // warp w's); lane m keeps worker m's and writes its scale and
@@ -376,19 +413,12 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
             if (m + 1 < M) add_worker(make_float2(scr.z, scr.w), xb);
         }
 
-        // 4. the mean's codec, the outer step and the stores
+        // 4. the mean's codec
         float v[PER];
 #pragma unroll
         for (int c = 0; c < PER; c += 4) {
-            const float4 q = *reinterpret_cast<const float4 *>(sv + e0 + c);
+            const float4 q = *reinterpret_cast<const float4 *>(sv + el(c));
             v[c] = q.x; v[c + 1] = q.y; v[c + 2] = q.z; v[c + 3] = q.w;
-        }
-        // this thread has read all of its staged chunks: their slots take
-        // the next block's copies while the rest of this block runs
-        if (nk < nblocks) {
-            stage_block<M, BF16, T>(stage, a, nstart, nlen,
-                                    nlen == kI8Block && a.nvec > 0 && (nstart % 8) == 0, t);
-            cp_commit();
         }
         float sum[PER];
 #pragma unroll
@@ -399,70 +429,86 @@ __global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
         const float fM = (float)M, rM = __frcp_rn(fM);
 #pragma unroll
         for (int i = 0; i < PER; ++i) sum[i] = div_by_scale(sum[i], fM, rM);
-        // elements beyond a short block hold 0 and do not move the maximum
+        // the previous block's bulk stores have read the tiles before any
+        // thread passes barrier 2 and rewrites them
+        if (t == 0) bulk_wait_read();
+        // barrier 2; elements beyond a short block hold 0 and do not move
+        // the maximum
         const float s = codec_scale(block_amax<PER, W>(sum, red1));
+        // every thread has read this block's staging: the next block's bulk
+        // copies go into the same buffer while the rest of this block runs
+        // (a short or unaligned next block is staged after the stores)
+        if (next_bulk && t == 0) stage_bulk(nk, nstart);
         const float rs = __frcp_rn(s);
         float gp[PER], vp[PER];
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
             const float dq = __fmul_rn(codec_code_fast(sum[i], s, rs), s);
-            const bool in = full || e0 + i < len;
+            const bool in = full || el(i) < len;
             if (in) b32 = fmaf(dq, dq, b32);
             outer_step(k, dq, g[i], v[i], gp[i], vp[i]);
             if (in) nf += not_finite(gp[i], vp[i]);
         }
-        if (full && vec) {
+
+        // 5. the stores
+        if (bulk) {
 #pragma unroll
             for (int c = 0; c < PER; c += 4) {
-                __stcs(reinterpret_cast<float4 *>(a.g + start + e0 + c),
-                       make_float4(gp[c], gp[c + 1], gp[c + 2], gp[c + 3]));
-                __stcs(reinterpret_cast<float4 *>(a.v + start + e0 + c),
-                       make_float4(vp[c], vp[c + 1], vp[c + 2], vp[c + 3]));
-            }
-            if constexpr (BF16) {
-                uint32_t w[NP];
-#pragma unroll
-                for (int j = 0; j < NP; ++j) w[j] = pack_bf16x2(gp[2 * j], gp[2 * j + 1]);
-#pragma unroll
-                for (int m = 0; m < M; ++m) {
-                    uint16_t *dst = reinterpret_cast<uint16_t *>(a.x[m]) + start + e0;
-                    if constexpr (PER == 4)
-                        __stcs(reinterpret_cast<uint2 *>(dst), make_uint2(w[0], w[1]));
-                    else
-                        __stcs(reinterpret_cast<uint4 *>(dst), make_uint4(w[0], w[1], w[2], w[3]));
+                if constexpr (BF16) {
+                    *reinterpret_cast<uint2 *>(ox + el(c) * 2) =
+                        make_uint2(pack_bf16x2(gp[c], gp[c + 1]), pack_bf16x2(gp[c + 2], gp[c + 3]));
                 }
-            } else {
-#pragma unroll
-                for (int m = 0; m < M; ++m)
-#pragma unroll
-                    for (int c = 0; c < PER; c += 4)
-                        __stcs(reinterpret_cast<float4 *>(
-                                   reinterpret_cast<float *>(a.x[m]) + start + e0 + c),
-                               make_float4(gp[c], gp[c + 1], gp[c + 2], gp[c + 3]));
+                if constexpr (GV || !BF16)
+                    *reinterpret_cast<float4 *>(og + el(c)) =
+                        make_float4(gp[c], gp[c + 1], gp[c + 2], gp[c + 3]);
+                if constexpr (GV)
+                    *reinterpret_cast<float4 *>(ov + el(c)) =
+                        make_float4(vp[c], vp[c + 1], vp[c + 2], vp[c + 3]);
+                if constexpr (!GV) {
+                    __stcs(reinterpret_cast<float4 *>(a.g + start + el(c)),
+                           make_float4(gp[c], gp[c + 1], gp[c + 2], gp[c + 3]));
+                    __stcs(reinterpret_cast<float4 *>(a.v + start + el(c)),
+                           make_float4(vp[c], vp[c + 1], vp[c + 2], vp[c + 3]));
+                }
             }
+            fence_proxy_async_smem();  // the tiles are read by bulk copies
+            pend = true;
+            pstart = start;
         } else {
 #pragma unroll
             for (int i = 0; i < PER; ++i) {
-                if (e0 + i >= len) continue;
-                a.g[start + e0 + i] = gp[i];
-                a.v[start + e0 + i] = vp[i];
+                const int e = el(i);
+                if (e >= len) continue;
+                a.g[start + e] = gp[i];
+                a.v[start + e] = vp[i];
 #pragma unroll
                 for (int m = 0; m < M; ++m) {
                     if constexpr (BF16)
-                        reinterpret_cast<__nv_bfloat16 *>(a.x[m])[start + e0 + i] =
+                        reinterpret_cast<__nv_bfloat16 *>(a.x[m])[start + e] =
                             __float2bfloat16_rn(gp[i]);
                     else
-                        reinterpret_cast<float *>(a.x[m])[start + e0 + i] = gp[i];
+                        reinterpret_cast<float *>(a.x[m])[start + e] = gp[i];
                 }
             }
         }
         b64 += (double)b32;  // at most PER terms per thread and block
         b32 = 0.f;
+        if (nk < nblocks && !next_bulk) stage_own(nstart, nlen);
 
         start = nstart;
         len = nlen;
     }
-    cp_wait<0>();
+    if (failed) {
+        if (t == 0) {
+            atomicExch(a.error, 1u);
+            // let the loads still in flight land before the CTA exits
+            if (in_flight) mbar_wait(bar, phase ^ 1, nullptr);
+        }
+    } else if (pend) {
+        __syncthreads();
+        if (t == 0) store_tiles(pstart);
+    }
+    if (t == 0) bulk_wait_all();
     if (since_flush > 0) flush();
     __syncthreads();
     double e64[M];
@@ -484,7 +530,8 @@ template <int M, bool BF16>
 cudaError_t fused_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
                          int max_grid, cudaStream_t stream, int *grid_out) {
     constexpr int T = fused_threads<M, BF16>();
-    constexpr size_t smem = stage_bytes<M, BF16, T>();
+    static_assert(fits<M, BF16, T>(), "fused INT8 staging exceeds shared memory");
+    constexpr size_t smem = fused_smem<M, BF16, T>();
     static PerDevice occ_cache;  // attribute set-up and occupancy, per device
     const int dev = PerDevice::device();
     int occ = occ_cache.get(dev);

@@ -17,6 +17,7 @@
 // still has in flight before the block exits.  The host reports the error.
 #pragma once
 
+#include "aloco_bulk.cuh"
 #include "aloco_sync_kernel.cuh"
 
 namespace aloco {
@@ -24,57 +25,6 @@ namespace aloco {
 constexpr int kTmaConsumers = kTmaTilePacks;       // 8 consumer warps
 constexpr int kTmaThreads = kTmaConsumers + 32;     // + 1 producer warp
 constexpr int kTmaMaxStages = 8;
-constexpr long long kTmaWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
-
-__device__ __forceinline__ uint32_t smem_addr(const void *p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count)
-                 : "memory");
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
-                 "r"(bytes)
-                 : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// Wait for the completion of the phase with the given parity.  Returns false
-// when the block aborted (abort != null) or the wait ran past the limit.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
-                                          const volatile int *abort) {
-    if (mbar_test(bar, parity)) return true;
-    const long long t0 = clock64();
-    while (!mbar_test(bar, parity)) {
-        if (abort && *abort) return false;
-        if (clock64() - t0 > kTmaWaitCycles) return false;
-    }
-    return true;
-}
-// Bulk copy global -> shared of `bytes` (multiple of 16, both addresses
-// 16-byte aligned), completing `bytes` of transaction count on `bar`.
-__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src,
-                                          uint32_t bytes, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes "
-        "[%0], [%1], %2, [%3];" ::"r"(dst),
-        "l"(src), "r"(bytes), "r"(bar)
-        : "memory");
-}
-
 // Bytes of one stage: theta and v tiles (fp32) and M replica tiles.
 template <bool BF16>
 __host__ __device__ constexpr uint32_t tma_gv_bytes() {

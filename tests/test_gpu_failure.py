@@ -1,9 +1,10 @@
 """Failure detection on the GPU without a GPU fault: every mbarrier wait of
-the bulk-copy pass is bounded, so a pipeline stage that never fills makes
-the round return an error status while every kernel finishes and the device
-stays usable.  The stall is requested through aloco_test_stall_tile, which
-makes the producer skip one tile's copies (its barrier is then never
-completed: a flag that nothing sets)."""
+the bulk-copy pass and of the fused INT8 round is bounded, so a stage that
+never fills makes the round return an error status while every kernel
+finishes and the device stays usable.  The stall is requested through
+aloco_test_stall_tile, which makes the issuing thread skip one tile's (or
+one codec block's) copies: its barrier is then never completed, a flag that
+nothing sets."""
 import time
 
 import pytest
@@ -67,3 +68,36 @@ def test_stall_hook_ignored_by_other_rounds():
     g, v, xs = gpu_inputs(w)
     st = A.sync(g, v, xs, opts=A.default_opts(pass_=A.PASS_BULK_COPY), **kw)
     assert st["status"] == A.OK and st["pass_used"] == A.PASS_BULK_COPY
+
+
+def test_stalled_int8_fused_block_is_reported_and_the_device_stays_usable():
+    w = W.small(1 << 22, 4, "bf16", seed=5)   # every codec block whole and aligned
+    kw = _kw(w)
+    fused = lambda: A.default_opts(pass_=A.PASS_INT8_FUSED)
+    g, v, xs = gpu_inputs(w)
+    st = A.sync_int8(g, v, xs, opts=fused(), **kw)
+    assert st["status"] == A.OK and st["pass_used"] == A.PASS_INT8_FUSED
+    block = 2 * st["grid"] + 5                # the third block of CTA 5
+    assert block < (w.numel + 4095) // 4096
+
+    g, v, xs = gpu_inputs(w)
+    A.test_stall_tile(block)
+    t0 = time.time()
+    st = A.sync_int8(g, v, xs, opts=fused(), raise_on_error=False, **kw)
+    took = time.time() - t0
+    assert st["status"] == A.ERR_CUDA
+    assert "timed out" in A.last_error()
+    assert 1.0 < took < 60.0, took
+    torch.cuda.synchronize()
+
+    # the next fused round runs and equals the split form bit for bit
+    g1, v1, x1 = gpu_inputs(w)
+    g2, v2, x2 = gpu_inputs(w)
+    st1 = A.sync_int8(g1, v1, x1, opts=fused(), **kw)
+    st2 = A.sync_int8(g2, v2, x2, opts=A.default_opts(pass_=A.PASS_INT8_SPLIT), **kw)
+    assert st1["status"] == st2["status"] == A.OK
+    assert st1["pass_used"] == A.PASS_INT8_FUSED
+    assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
+    assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))
+    for a_, b_ in zip(x1, x2):
+        assert torch.equal(a_.view(torch.int16), b_.view(torch.int16))
