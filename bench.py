@@ -43,7 +43,7 @@ UNIT = "rounds/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 PASSES = {"auto": 0, "registers": 1, "bulk_copy": 2, "int8_split": 3,
-          "int8_fused": 4}
+          "int8_fused": 4, "tile": 5}
 
 
 def workloads_by_name():
@@ -83,6 +83,7 @@ def hbm_peak():
 KERNEL_SOURCES = {
     "sync_kernel": ("aloco_sync_kernel.cuh", "aloco_sync_f32.cu",
                     "aloco_sync_bf16.cu"),
+    "sync_tile_kernel": ("aloco_sync_kernel.cuh", "aloco_bulk.cuh", "aloco_sync_tile.cu"),
     "sync_tma_kernel": ("aloco_sync_kernel.cuh", "aloco_bulk.cuh", "aloco_sync_tma.cuh",
                         "aloco_sync_tma_f32.cu", "aloco_sync_tma_bf16.cu"),
     "int8_split_kernels": ("aloco_sync_kernel.cuh", "aloco_int8.cuh",
@@ -415,7 +416,7 @@ def run_cuda(args, w):
         step_ms.append(ev[k][0].elapsed_time(ev[k][1]))
 
     kernel_name = {2: "sync_tma_kernel", 3: "int8_split_kernels",
-                   4: "int8_fused_kernel"}.get(st_first.get("pass_used"),
+                   4: "int8_fused_kernel", 5: "sync_tile_kernel"}.get(st_first.get("pass_used"),
                                                "sync_kernel")
     ms_step = statistics.mean(step_ms)
     ms_step = reduce_max(ms_step, world, device)

@@ -105,16 +105,22 @@ typedef enum {
     ALOCO_CORR_NONE = 2
 } aloco_corr_mode;
 
-/* The two implementations of the fused pass.  Both compute the same round
- * with the same arithmetic; they differ in how data reaches the SMs.
+/* The implementations of the fused pass.  All compute the same round with
+ * the same per-element arithmetic (theta', v' and the replicas agree bit
+ * for bit); they differ in how data reaches the SMs.
  *   REGISTERS  every thread streams 16-byte loads of theta, v and the
  *              replicas straight into registers (any M, any alignment);
  *   BULK_COPY  a producer warp per SM stages 4-8 KB tiles of every array in
  *              a shared-memory ring with cp.async.bulk and mbarriers, and
  *              consumer warps compute from shared memory (M <= 16, 16-byte
  *              aligned buffers; otherwise REGISTERS runs);
- *   AUTO       the faster of the two as measured on GB300: at present the
- *              register-streaming pass for every (M, dtype).
+ *   TILE       CTAs stage whole blocks of every array with cp.async.bulk,
+ *              write theta' once to a shared-memory tile and store the
+ *              replica reset as M bulk copies of it (M <= 8, 16-byte
+ *              aligned buffers, N >= 4096; otherwise REGISTERS runs);
+ *   AUTO       the fastest as measured on GB300 for (M, dtype, N): TILE
+ *              from 2^27 parameters for bf16 replicas and for fp32 with
+ *              M = 1 or 5..8, else REGISTERS.
  * The INT8-communicated round (aloco_sync_int8) has two forms of its own:
  *   INT8_SPLIT a block-scale kernel, then an apply kernel that reads the
  *              replicas again (any M <= 16);
@@ -123,13 +129,14 @@ typedef enum {
  *              (M <= 8; ALOCO_ERR_ARG otherwise);
  *   AUTO       the form measured faster on GB300 for (M, dtype).
  * aloco_sync / aloco_sync_ex reject the INT8 values and aloco_sync_int8 the
- * REGISTERS / BULK_COPY values with ALOCO_ERR_ARG. */
+ * REGISTERS / BULK_COPY / TILE values with ALOCO_ERR_ARG. */
 typedef enum {
     ALOCO_PASS_AUTO = 0,
     ALOCO_PASS_REGISTERS = 1,
     ALOCO_PASS_BULK_COPY = 2,
     ALOCO_PASS_INT8_SPLIT = 3,
-    ALOCO_PASS_INT8_FUSED = 4
+    ALOCO_PASS_INT8_FUSED = 4,
+    ALOCO_PASS_TILE = 5
 } aloco_pass;
 
 /* Options.  aloco_default_opts() fills the paper's settings

@@ -18,6 +18,7 @@ SCHED_COSINE, SCHED_CONSTANT, SCHED_LINEAR = 0, 1, 2
 CORR_FULL, CORR_MOMENTUM_ONLY, CORR_NONE = 0, 1, 2
 PASS_AUTO, PASS_REGISTERS, PASS_BULK_COPY = 0, 1, 2
 PASS_INT8_SPLIT, PASS_INT8_FUSED = 3, 4
+PASS_TILE = 5
 
 OK = 0
 ERR_ARG = -1

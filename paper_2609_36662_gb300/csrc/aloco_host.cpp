@@ -111,7 +111,7 @@ int correction_impl(const aloco_schedule_t *sched, int64_t step,
     if (!std::isfinite(outer_lr)) return fail(ALOCO_ERR_ARG, "outer_lr must be finite");
     if (o.blocks_per_sm < 0)
         return fail(ALOCO_ERR_ARG, "blocks_per_sm must be >= 0");
-    if (o.pass < ALOCO_PASS_AUTO || o.pass > ALOCO_PASS_INT8_FUSED)
+    if (o.pass < ALOCO_PASS_AUTO || o.pass > ALOCO_PASS_TILE)
         return fail(ALOCO_ERR_ARG, "unknown pass %d", o.pass);
     if (o.mode != ALOCO_CORR_FULL && o.mode != ALOCO_CORR_MOMENTUM_ONLY &&
         o.mode != ALOCO_CORR_NONE)
@@ -277,7 +277,7 @@ GetAddressRangeFn address_range_fn() {
 // Helpers with external linkage: also used by the allocation-free entry
 // point (aloco_noalloc.cu).
 // Testing hook of aloco_test_stall_tile: consumed by the calling thread's
-// next bulk-copy or fused INT8 round.
+// next bulk-copy, tile or fused INT8 round.
 thread_local int64_t t_test_stall_tile1 = 0;
 
 namespace aloco {
@@ -289,13 +289,27 @@ bool use_int8_fused(int pass, int M, aloco_dtype dtype) {
     return true;  // AUTO
 }
 
+bool use_tile(int pass, int M, aloco_dtype dtype, int64_t n, int64_t nvec) {
+    if (!sync_tile_fits(M, n, nvec)) return false;
+    if (pass == ALOCO_PASS_TILE) return true;
+    if (pass != ALOCO_PASS_AUTO) return false;
+    // AUTO, as measured on GB300 (fraction of the measured copy peak): from
+    // 2^27 parameters the tile pass leads for bf16 replicas (0.97-0.98
+    // against 0.94) and for fp32 with M = 1 or M >= 5 (0.96-0.98 against
+    // 0.94-0.95); at fp32 M = 2..4 the two passes tie within 0.5 %.  On
+    // smaller rounds the CTAs of the tile pass move through their blocks in
+    // step, so HBM idles while they compute, and the register pass leads.
+    if (n < ((int64_t)1 << 27)) return false;
+    return dtype == ALOCO_BF16 || M == 1 || M >= 5;
+}
+
 bool use_tma(int pass, int M, aloco_dtype dtype, int64_t nvec) {
     if (M < 1 || M > 16 || nvec < kTmaTilePacks) return false;
     if (pass == ALOCO_PASS_BULK_COPY) return true;
     if (pass == ALOCO_PASS_REGISTERS) return false;
     // AUTO: on GB300 the tuned register-streaming pass matched or beat the
     // bulk-copy ring on every full-size workload measured (150M x 8 fp32:
-    // 95.9 % vs 93.6 % of copy bandwidth; 3B x 8 bf16: 95.9 % vs 95.7 %).
+    // 0.94 against 0.92 of the measured copy peak; 3B x 8 bf16: 0.94 each).
     (void)dtype;
     return false;
 }
@@ -457,7 +471,8 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     if (dtype != ALOCO_F32 && dtype != ALOCO_BF16)
         return fail(ALOCO_ERR_ARG, "unknown replica dtype %d", (int)dtype);
     const bool int8_pass = o.pass == ALOCO_PASS_INT8_SPLIT || o.pass == ALOCO_PASS_INT8_FUSED;
-    if (int8 ? (o.pass == ALOCO_PASS_REGISTERS || o.pass == ALOCO_PASS_BULK_COPY)
+    if (int8 ? (o.pass == ALOCO_PASS_REGISTERS || o.pass == ALOCO_PASS_BULK_COPY ||
+                o.pass == ALOCO_PASS_TILE)
              : int8_pass)
         return fail(ALOCO_ERR_ARG, "pass %d does not apply to this round", o.pass);
     if (int8 && o.pass == ALOCO_PASS_INT8_FUSED && !aloco::int8_fused_fits(M, dtype))
@@ -546,9 +561,10 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
 
     const int64_t work = a.nvec > 0 ? a.nvec : a.n;
     aloco::LaunchPlan plan;
-    const bool tma = !int8 && aloco::use_tma(o.pass, M, dtype, a.nvec);
+    const bool tile = !int8 && aloco::use_tile(o.pass, M, dtype, a.n, a.nvec);
+    const bool tma = !int8 && !tile && aloco::use_tma(o.pass, M, dtype, a.nvec);
     const bool fused = int8 && aloco::use_int8_fused(o.pass, M, dtype);
-    if (fused) {
+    if (fused || tile) {
         plan.grid = 0;
         plan.block = 0;
         plan.kernel = nullptr;
@@ -583,7 +599,7 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     a.n_tiles = plan.tiles;
     a.stages = plan.stages;
     a.error = ws->error;
-    if (tma || fused) {
+    if (tma || fused || tile) {
         a.test_stall_tile1 = t_test_stall_tile1;
         t_test_stall_tile1 = 0;
     }
@@ -597,6 +613,8 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     if (fused) {
         e = aloco::launch_int8_fused(a, P, dtype, ws->sm_count, ws->max_grid, stream,
                                      &plan.grid);
+    } else if (tile) {
+        e = aloco::launch_sync_tile(a, dtype, ws->sm_count, ws->max_grid, stream, &plan.grid);
     } else if (int8) {
         double *e_rows = reinterpret_cast<double *>(ws->i8);
         unsigned *bmax = reinterpret_cast<unsigned *>(
@@ -632,6 +650,7 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     st->grid = plan.grid;
     st->pass_used = fused ? ALOCO_PASS_INT8_FUSED
                     : int8 ? ALOCO_PASS_INT8_SPLIT
+                    : tile ? ALOCO_PASS_TILE
                     : tma  ? ALOCO_PASS_BULK_COPY
                            : ALOCO_PASS_REGISTERS;
     if (o.time_kernel) {

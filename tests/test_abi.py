@@ -227,7 +227,7 @@ def test_pass_values_are_checked_against_the_round(lib):
     s = A.Schedule.make()
     base = 1 << 40
     xs = [base + (k + 2) * (1 << 22) for k in range(2)]
-    for p in (A.PASS_INT8_SPLIT, A.PASS_INT8_FUSED, 5, -1):
+    for p in (A.PASS_INT8_SPLIT, A.PASS_INT8_FUSED, 6, -1):
         for noalloc in (False, True):
             rc, _ = A.sync_ptrs(base, base + (1 << 22), xs, 1000, A.F32, 150,
                                 100, 4000, s, 0.7, 0.9,
@@ -245,7 +245,7 @@ def test_pass_values_are_checked_against_the_round(lib):
                                    0.7, 0.9, None, 0,
                                    ctypes.byref(A.default_opts(pass_=p)),
                                    ctypes.byref(st))
-    for p in (A.PASS_REGISTERS, A.PASS_BULK_COPY):
+    for p in (A.PASS_REGISTERS, A.PASS_BULK_COPY, A.PASS_TILE):
         assert int8(2, A.F32, p) == A.ERR_ARG
     assert int8(9, A.F32, A.PASS_INT8_FUSED) == A.ERR_ARG
     assert int8(9, A.BF16, A.PASS_INT8_FUSED) == A.ERR_ARG

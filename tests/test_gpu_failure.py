@@ -101,3 +101,33 @@ def test_stalled_int8_fused_block_is_reported_and_the_device_stays_usable():
     assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))
     for a_, b_ in zip(x1, x2):
         assert torch.equal(a_.view(torch.int16), b_.view(torch.int16))
+
+
+def test_stalled_tile_pass_block_is_reported_and_the_device_stays_usable():
+    w = W.small(1 << 22, 3, "f32", seed=5)
+    kw = _kw(w)
+    tile = lambda: A.default_opts(pass_=A.PASS_TILE)
+    g, v, xs = gpu_inputs(w)
+    st = A.sync(g, v, xs, opts=tile(), **kw)
+    assert st["status"] == A.OK and st["pass_used"] == A.PASS_TILE
+    block = 3 * st["grid"] + 11            # the fourth block of CTA 11
+    assert block < w.numel // 4096
+
+    g, v, xs = gpu_inputs(w)
+    A.test_stall_tile(block)
+    t0 = time.time()
+    st = A.sync(g, v, xs, opts=tile(), raise_on_error=False, **kw)
+    took = time.time() - t0
+    assert st["status"] == A.ERR_CUDA
+    assert "timed out" in A.last_error()
+    assert 1.0 < took < 60.0, took
+    torch.cuda.synchronize()
+
+    g1, v1, x1 = gpu_inputs(w)
+    g2, v2, x2 = gpu_inputs(w)
+    st1 = A.sync(g1, v1, x1, opts=tile(), **kw)
+    st2 = A.sync(g2, v2, x2, opts=A.default_opts(pass_=A.PASS_REGISTERS), **kw)
+    assert st1["status"] == st2["status"] == A.OK
+    assert st1["pass_used"] == A.PASS_TILE
+    assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
+    assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))

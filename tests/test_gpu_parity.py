@@ -14,7 +14,7 @@ import oracle as O
 from paper_2609_36662_gb300 import aloco as A
 from paper_2609_36662_gb300 import workloads as W
 
-from _parity import (assert_corr, assert_field, assert_field_after_chain,
+from _parity import (RTOL_STAT, assert_corr, assert_field, assert_field_after_chain,
                      assert_stats, compare_round, gpu_inputs,
                      oracle_chain_replicas,
                      run_gpu_round, run_oracle_round, schedule_pair,
@@ -70,16 +70,17 @@ MEDIUM = [(1_000_003, m, dt) for m in (1, 3, 4, 8, 16, 17, 32)
           for dt in ("f32", "bf16")]
 
 
-PASSES = [A.PASS_REGISTERS, A.PASS_BULK_COPY]
-PASS_IDS = ["registers", "bulk_copy"]
+PASSES = [A.PASS_REGISTERS, A.PASS_BULK_COPY, A.PASS_TILE]
+PASS_IDS = ["registers", "bulk_copy", "tile"]
 
 
 @pytest.mark.parametrize("pass_", PASSES, ids=PASS_IDS)
 @pytest.mark.parametrize("N,M,dt", SMALL + MEDIUM)
 def test_round_matches_oracle(N, M, dt, pass_):
-    """Both fused passes against the oracle.  The bulk-copy pass serves M <=
-    16 with 16-byte aligned buffers and at least one whole tile; other
-    rounds fall back to the register-streaming pass."""
+    """Every fused pass against the oracle.  The bulk-copy pass serves M <=
+    16 with 16-byte aligned buffers and at least one whole tile, the tile
+    pass M <= 8 with aligned buffers and N >= 4096; other rounds fall back
+    to the register-streaming pass."""
     w = W.small(N, M, dt, seed=N % 97 + M)
     g, v, xs = gpu_inputs(w)
     v.normal_(0, 1e-3)          # carried momentum
@@ -87,8 +88,10 @@ def test_round_matches_oracle(N, M, dt, pass_):
     st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0],
                        opts=A.default_opts(pass_=pass_))
     assert st["status"] == A.OK
-    tma_ok = M <= 16 and N * (4 if dt == "f32" else 2) >= 256 * 16
-    assert st["pass_used"] == (pass_ if tma_ok else A.PASS_REGISTERS)
+    runs = {A.PASS_REGISTERS: True,
+            A.PASS_BULK_COPY: M <= 16 and N * (4 if dt == "f32" else 2) >= 256 * 16,
+            A.PASS_TILE: M <= 8 and N >= 4096}[pass_]
+    assert st["pass_used"] == (pass_ if runs else A.PASS_REGISTERS)
     compare_round(w, st, orc, g, v, xs)
 
 
@@ -294,3 +297,30 @@ def test_momentum_carried_across_rounds(dt):
         assert_field(g.cpu().numpy(), orc["g"], f"theta' round {k}")
         assert_field(v.cpu().numpy(), orc["v"], f"v' round {k}")
         v_o = orc["v"].astype(np.float32)
+
+
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 5, 6, 7, 8])
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+def test_tile_pass_equals_register_pass_bit_for_bit(M, dt):
+    """The tile pass runs the register pass's per-element arithmetic:
+    theta', v' and every replica agree bit for bit, on whole blocks and on
+    the element-wise tail; the statistics agree within their tolerance."""
+    w = W.small(3 * 2048 * 37 + 1234, M, dt, seed=40 + M)
+    out = []
+    for p in (A.PASS_TILE, A.PASS_REGISTERS):
+        g, v, xs = gpu_inputs(w)
+        v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(2))
+        st = run_gpu_round(g, v, xs, w, w.start_step, w.H_sel[0],
+                           opts=A.default_opts(pass_=p))
+        assert st["status"] == A.OK and st["pass_used"] == p
+        out.append((st, g, v, xs))
+    (s1, g1, v1, x1), (s2, g2, v2, x2) = out
+    assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
+    assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))
+    for a_, b_ in zip(x1, x2):
+        assert torch.equal(a_.view(torch.int16) if dt == "bf16" else a_.view(torch.int32),
+                           b_.view(torch.int16) if dt == "bf16" else b_.view(torch.int32))
+    assert s1["D"] == pytest.approx(s2["D"], rel=RTOL_STAT)
+    assert s1["mean_sq_norm"] == pytest.approx(s2["mean_sq_norm"], rel=RTOL_STAT)
+    for m in range(M):
+        assert s1["drift"][m] == pytest.approx(s2["drift"][m], rel=RTOL_STAT)
