@@ -243,6 +243,12 @@ int aloco_sync(float *global, float *momentum, void *const *locals,
  * accesses.  Returns ALOCO_ERR_NONFINITE when some theta' or v' is NaN/Inf
  * (outputs and statistics are still written; the paper's controller treats
  * a non-finite statistic as a reduction signal, App. A.2).
+ * Completion: the call returns once the round's last block has published
+ * the statistics, which it does after every block has written its outputs.
+ * The kernel may still be retiring on opts->stream; work queued there
+ * later runs after it, and work on other streams that must follow the
+ * round should wait on that stream.  The INT8 round (aloco_sync_int8)
+ * behaves the same way.
  * Thread safety: calls for the same device are serialised internally. */
 int aloco_sync_ex(float *global, float *momentum, void *const *locals,
                   size_t N, int M, aloco_dtype dtype, int64_t H_sel,

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -180,6 +181,11 @@ struct Workspace {
     char *i8 = nullptr;                   // INT8 round scratch (grown on demand)
     size_t i8_cap = 0;
     double *host = nullptr;               // pinned readback of totals + nf
+    // device-mapped page-locked page the round kernels publish their totals
+    // and sequence number to (kTotals + 1 slots), and its device address
+    double *stats_host = nullptr;
+    double *stats_dev = nullptr;
+    unsigned long long seq = 0;           // rounds launched on this workspace
     cudaEvent_t ev0 = nullptr, ev1 = nullptr;
     // host-memory round (aloco_sync_host): staging slots and per-chunk totals
     char *hs = nullptr;                   // device, grown on demand
@@ -241,6 +247,13 @@ int ensure_ready(Workspace *ws, int device) {
     ws->ticket = (unsigned int *)p;
     e = cudaMemset(ws->dev, 0, bytes);
     if (e == cudaSuccess) e = cudaMallocHost((void **)&ws->host, kHostSlots * sizeof(double));
+    if (e == cudaSuccess)
+        e = cudaHostAlloc((void **)&ws->stats_host, (kTotals + 1) * sizeof(double),
+                          cudaHostAllocMapped);
+    if (e == cudaSuccess) {
+        std::memset(ws->stats_host, 0, (kTotals + 1) * sizeof(double));
+        e = cudaHostGetDevicePointer((void **)&ws->stats_dev, ws->stats_host, 0);
+    }
     if (e == cudaSuccess) e = cudaEventCreate(&ws->ev0);
     if (e == cudaSuccess) e = cudaEventCreate(&ws->ev1);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -250,6 +263,29 @@ int ensure_ready(Workspace *ws, int device) {
     }
     ws->device = device;
     ws->ready = true;
+    return ALOCO_OK;
+}
+
+// Wait until the round kernel has published round `seq` to `page` (see
+// SyncArgs::stats_out).  The last block publishes after every block's
+// outputs are written, so on return the outputs are complete, and work
+// queued later on the stream runs after the kernel.  The stream is polled
+// every few hundred reads: a launch that fails or ends without publishing
+// returns an error instead of waiting on.
+int wait_published(const double *page, unsigned long long seq, cudaStream_t stream) {
+    const volatile unsigned long long *flag =
+        reinterpret_cast<const volatile unsigned long long *>(page + aloco::kSeqSlot);
+    for (unsigned it = 1;; ++it) {
+        if (*flag == seq) break;
+        if ((it & 255) == 0) {
+            const cudaError_t q = cudaStreamQuery(stream);
+            if (q == cudaErrorNotReady) continue;
+            if (q != cudaSuccess) return cuda_fail(q, "round");
+            if (*flag == seq) break;
+            return fail(ALOCO_ERR_CUDA, "the round ended without publishing its statistics");
+        }
+    }
+    std::atomic_thread_fence(std::memory_order_acquire);
     return ALOCO_OK;
 }
 
@@ -599,6 +635,8 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     a.n_tiles = plan.tiles;
     a.stages = plan.stages;
     a.error = ws->error;
+    a.stats_out = ws->stats_dev;
+    a.seq = ++ws->seq;
     if (tma || fused || tile) {
         a.test_stall_tile1 = t_test_stall_tile1;
         t_test_stall_tile1 = 0;
@@ -629,16 +667,12 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     if (e != cudaSuccess) return cuda_fail(e, "fused sync launch");
     if (o.time_kernel && (e = cudaEventRecord(ws->ev1, stream)) != cudaSuccess)
         return cuda_fail(e, "cudaEventRecord");
-    e = cudaMemcpyAsync(ws->host, ws->totals, kTotals * sizeof(double),
-                        cudaMemcpyDeviceToHost, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "statistics readback");
-    e = cudaStreamSynchronize(stream);
-    if (e != cudaSuccess) return cuda_fail(e, "round");
+    if ((rc = wait_published(ws->stats_host, a.seq, stream)) != ALOCO_OK) return rc;
 
     unsigned long long nf;
-    std::memcpy(&nf, ws->host + aloco::kNfSlot, sizeof nf);
+    std::memcpy(&nf, ws->stats_host + aloco::kNfSlot, sizeof nf);
     unsigned int perr;
-    std::memcpy(&perr, ws->host + aloco::kErrorSlot, sizeof perr);
+    std::memcpy(&perr, ws->stats_host + aloco::kErrorSlot, sizeof perr);
     if (perr != 0) {
         cudaMemsetAsync(ws->error, 0, sizeof(unsigned int), stream);
         cudaStreamSynchronize(stream);
@@ -646,7 +680,8 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
         return fail(ALOCO_ERR_CUDA,
                     "bulk-copy pipeline wait timed out; outputs are incomplete");
     }
-    finalize_stats(ws->host, nf, M, o.eps, int8 ? 1.0 : 1.0 / ((double)M * (double)M), st);
+    finalize_stats(ws->stats_host, nf, M, o.eps, int8 ? 1.0 : 1.0 / ((double)M * (double)M),
+                   st);
     st->grid = plan.grid;
     st->pass_used = fused ? ALOCO_PASS_INT8_FUSED
                     : int8 ? ALOCO_PASS_INT8_SPLIT
@@ -655,7 +690,8 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
                            : ALOCO_PASS_REGISTERS;
     if (o.time_kernel) {
         float ms = -1.f;
-        if (cudaEventElapsedTime(&ms, ws->ev0, ws->ev1) == cudaSuccess)
+        if (cudaEventSynchronize(ws->ev1) == cudaSuccess &&
+            cudaEventElapsedTime(&ms, ws->ev0, ws->ev1) == cudaSuccess)
             st->kernel_ms = ms;
         else
             cudaGetLastError();
@@ -1277,6 +1313,7 @@ void aloco_shutdown(void) {
         if (ws->ev0) cudaEventDestroy(ws->ev0);
         if (ws->ev1) cudaEventDestroy(ws->ev1);
         if (ws->host) cudaFreeHost(ws->host);
+        if (ws->stats_host) cudaFreeHost(ws->stats_host);
         if (ws->dev) cudaFree(ws->dev);
         if (ws->i8) cudaFree(ws->i8);
         ws->i8 = nullptr;
@@ -1299,6 +1336,8 @@ void aloco_shutdown(void) {
         ws->hs_in = ws->hs_out = nullptr;
         ws->ev0 = ws->ev1 = nullptr;
         ws->host = nullptr;
+        ws->stats_host = nullptr;
+        ws->stats_dev = nullptr;
         ws->dev = nullptr;
         ws->ready = false;
     }

@@ -63,6 +63,12 @@ struct SyncArgs {
     unsigned int *error;            // set to 1 if a pipeline wait timed out
     int64_t test_stall_tile1;       // testing only: 1 + the index of a tile whose
                                     // copies the producer skips (0 = none)
+    // Statistics published to the host (null: not published).  The last
+    // block writes the totals block (kTotalsSlots values) to this
+    // device-mapped page-locked host memory, then, after a system-scope
+    // fence, `seq` to slot kSeqSlot.
+    double *stats_out;
+    unsigned long long seq;
 };
 
 // Slots of the totals block read back after a round (8 bytes each): M + 1
@@ -70,6 +76,8 @@ struct SyncArgs {
 constexpr int kTotalsSlots = ALOCO_MAX_WORKERS + 3;
 constexpr int kNfSlot = ALOCO_MAX_WORKERS + 1;
 constexpr int kErrorSlot = ALOCO_MAX_WORKERS + 2;
+// The published round sequence number follows the totals block.
+constexpr int kSeqSlot = kTotalsSlots;
 
 // Shared memory the bulk-copy pass may use for its ring (bytes), and the
 // packs of one tile (one per consumer thread).

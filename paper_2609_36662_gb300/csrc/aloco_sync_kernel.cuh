@@ -267,6 +267,18 @@ __device__ __forceinline__ void reduce_and_finish(const SyncArgs &a, int M,
         *a.nf_total = t;
         *a.ticket = 0u;  // ready for the next launch
     }
+    if (a.stats_out) {
+        // publish the totals block to the host, then the round's number
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            volatile double *out = a.stats_out;
+            for (int p = 0; p < np; ++p) out[p] = __ldcg(a.totals + p);
+            out[kNfSlot] = __longlong_as_double((long long)__ldcg(a.nf_total));
+            out[kErrorSlot] = __ldcg(a.totals + kErrorSlot);
+            __threadfence_system();
+            reinterpret_cast<volatile unsigned long long *>(a.stats_out)[kSeqSlot] = a.seq;
+        }
+    }
 }
 
 // Minimum resident blocks per SM the register allocator must allow (it
