@@ -103,9 +103,9 @@ def kernel_source_hash(kernel: str) -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload: str, kernel: str):
-    """DRAM bytes per launch of the fused pass from the committed ncu
-    summary, if it was taken on the current kernel source."""
+def recorded_entry(workload: str, kernel: str):
+    """The committed ncu record of this kernel on this workload, if it was
+    taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -115,7 +115,24 @@ def recorded_traffic(workload: str, kernel: str):
     entry = rec.get(f"{workload}/{kernel}")
     if not entry or entry.get("kernel_hash") != kernel_source_hash(kernel):
         return None
-    return entry.get("dram_bytes_per_launch")
+    return entry
+
+
+def recorded_traffic(workload: str, kernel: str):
+    """DRAM bytes per launch of the fused pass from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    entry = recorded_entry(workload, kernel)
+    return entry.get("dram_bytes_per_launch") if entry else None
+
+
+def recorded_occupancy(workload: str, kernel: str):
+    """Achieved occupancy (ncu sm__warps_active, % of the SM's warp slots)
+    from the same record, with the case it was measured on."""
+    entry = recorded_entry(workload, kernel)
+    if not entry or entry.get("warps_active_pct") is None:
+        return None
+    return {"warps_active_pct": entry["warps_active_pct"],
+            "measured_on": entry["measured_on"].split(":")[0]}
 
 
 # ------------------------------------------------------------------ clocks
@@ -521,6 +538,7 @@ def run_cuda(args, w):
                          "peak_source": peak_kind,
                          "traffic": recorded_traffic(w.name, kernel_name),
                          "kernel": kernel_name,
+                         "occupancy": recorded_occupancy(w.name, kernel_name),
                          "algorithmic_bytes_per_launch": w.bytes_per_round()},
             "cpu_baseline": cpu_baseline,
             "e2e": e2e,
@@ -839,6 +857,8 @@ def run_adamw(args, w):
                                      if norms is None else None),
                          "kernel": ("adamw_kernels" if norms is None
                                     else "adamw_update_kernel"),
+                         "occupancy": (recorded_occupancy(w.name, "adamw_kernels")
+                                       if norms is None else None),
                          "algorithmic_bytes_per_launch": adamw_bytes(w)},
             "grad_norms": st["grad_norm"], "clip": st["clip"],
             "cpu_baseline": cpu_baseline, "e2e": e2e,
