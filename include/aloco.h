@@ -116,7 +116,7 @@ typedef enum {
  *              aligned buffers; otherwise REGISTERS runs);
  *   TILE       CTAs stage whole blocks of every array with cp.async.bulk,
  *              write theta' once to a shared-memory tile and store the
- *              replica reset as M bulk copies of it (M <= 8, 16-byte
+ *              replica reset as M bulk copies of it (M <= 16, 16-byte
  *              aligned buffers, N >= 4096; otherwise REGISTERS runs);
  *   AUTO       the fastest as measured on GB300 for (M, dtype, N): TILE
  *              from 2^27 parameters for bf16 replicas and for fp32 with

@@ -335,8 +335,12 @@ bool use_tile(int pass, int M, aloco_dtype dtype, int64_t n, int64_t nvec) {
     // 0.94-0.95); at fp32 M = 2..4 the two passes tie within 0.5 %.  On
     // smaller rounds the CTAs of the tile pass move through their blocks in
     // step, so HBM idles while they compute, and the register pass leads.
+    // M = 9..16 from 2^27 too: fp32 0.99-1.00 against 0.95-0.97 (M >= 12),
+    // bf16 0.96-0.97 against 0.955-0.963 (M <= 12); bf16 M >= 13 spills
+    // registers in the tile pass and stays on the register pass.
     if (n < ((int64_t)1 << 27)) return false;
-    return dtype == ALOCO_BF16 || M == 1 || M >= 5;
+    if (dtype == ALOCO_BF16) return M <= 12;
+    return M == 1 || M >= 5;
 }
 
 bool use_tma(int pass, int M, aloco_dtype dtype, int64_t nvec) {

@@ -114,7 +114,7 @@ cudaError_t plan_sync_tma_bf16(int M, int64_t nvec, int sm_count,
 // Whether a round of M workers (dtype) uses the bulk-copy pass, given the
 // requested aloco_pass.
 bool use_tma(int pass, int M, aloco_dtype dtype, int64_t nvec);
-// The tile pass (aloco_sync_tile.cu): M <= 8, aligned buffers, at least one
+// The tile pass (aloco_sync_tile.cu): M <= 16, aligned buffers, at least one
 // whole block.
 bool sync_tile_fits(int M, int64_t n, int64_t nvec);
 bool use_tile(int pass, int M, aloco_dtype dtype, int64_t n, int64_t nvec);

@@ -1,5 +1,5 @@
 // Fused outer-synchronisation pass staged through shared memory by bulk
-// copies (the "tile" pass; M <= 8, 16-byte aligned buffers).
+// copies (the "tile" pass; M <= 16, 16-byte aligned buffers).
 //
 // The arithmetic per element is the register-streaming pass's (Algorithm 1:
 // Delta_m = theta - x_m summed in worker order; the drift energies and
@@ -35,7 +35,7 @@ namespace aloco {
 
 namespace {
 
-constexpr int kTileMaxM = 8;
+constexpr int kTileMaxM = 16;
 constexpr int kTileFlushBlocks = 8;
 constexpr size_t kTileSmemPerSm = 233472;   // shared memory of one SM
 constexpr size_t kTileSmemReserved = 1024;  // reserved by the system per CTA
@@ -53,19 +53,21 @@ constexpr size_t kTileSmemReserved = 1024;  // reserved by the system per CTA
 #define ALOCO_TILE_NOGV 0
 #endif
 #ifndef ALOCO_TILE_CTAS
-#define ALOCO_TILE_CTAS 0  // CTAs per SM (0: 1024 / T, 64 registers a thread)
+#define ALOCO_TILE_CTAS 0  // CTAs per SM (0: the table in tile_ctas)
 #endif
 
 template <bool BF16>
 __host__ __device__ constexpr int tile_es() { return BF16 ? 2 : 4; }
-// CTAs per SM the shared-memory budget is planned for
-template <int T>
+// CTAs per SM the shared-memory budget is planned for: 1024 threads per SM
+// (64 registers a thread), except fp32 with M > 8, whose 2048-element stage
+// fits one 512-thread CTA per SM
+template <int M, bool BF16, int T>
 __host__ __device__ constexpr int tile_ctas() {
-    return ALOCO_TILE_CTAS ? ALOCO_TILE_CTAS : 1024 / T;
+    return ALOCO_TILE_CTAS ? ALOCO_TILE_CTAS : (!BF16 && M > 8) ? 1 : 1024 / T;
 }
-template <int T>
+template <int M, bool BF16, int T>
 __host__ __device__ constexpr size_t tile_budget() {
-    return kTileSmemPerSm / tile_ctas<T>() - kTileSmemReserved;
+    return kTileSmemPerSm / tile_ctas<M, BF16, T>() - kTileSmemReserved;
 }
 // static shared memory: energy rows, the final reduction, barriers (bound)
 template <int M, int T>
@@ -88,7 +90,7 @@ __host__ __device__ constexpr size_t tile_smem() {
 }
 template <int M, bool BF16, int T, int NS, bool GV>
 __host__ __device__ constexpr bool tile_fit() {
-    return tile_smem<M, BF16, T, NS, GV>() + tile_static<M, T>() <= tile_budget<T>();
+    return tile_smem<M, BF16, T, NS, GV>() + tile_static<M, T>() <= tile_budget<M, BF16, T>();
 }
 // Shapes measured on GB300 (fraction of the measured copy peak, rounds of
 // 1.4e8 - 5e8 parameters):
@@ -98,14 +100,20 @@ __host__ __device__ constexpr bool tile_fit() {
 //     0.95-0.97;
 //   bf16 M >= 5: two 512-thread CTAs per SM with one stage, so that the
 //     fp32 output tiles fit, 0.97-0.98 against 0.93-0.97.
+//   M = 9..16: 512-thread CTAs with one stage (one CTA per SM for fp32,
+//     two for bf16); fp32 0.99-1.00 for M = 12..16 against 0.95-0.97 for
+//     the register pass, bf16 0.96-0.97 for M = 9..12 against 0.955-0.963.
 template <int M, bool BF16>
 __host__ __device__ constexpr int tile_threads() {
-    return ALOCO_TILE_T ? ALOCO_TILE_T : !BF16 ? 1024 : (M <= 4 ? 256 : 512);
+    return ALOCO_TILE_T ? ALOCO_TILE_T
+           : M > 8      ? 512
+           : !BF16      ? 1024
+                        : (M <= 4 ? 256 : 512);
 }
 template <int M, bool BF16, int T>
 __host__ __device__ constexpr int tile_stages() {
     return ALOCO_TILE_NS ? ALOCO_TILE_NS
-           : BF16 ? 1
+           : (BF16 || M > 8) ? 1
            : (tile_fit<M, BF16, T, 2, false>() ? 2 : 1);
 }
 template <int M, bool BF16, int T, int NS>
@@ -116,7 +124,7 @@ __host__ __device__ constexpr bool tile_gv() {
 }  // namespace
 
 template <int M, bool BF16, int T, int NS>
-__global__ void __launch_bounds__(T, (tile_ctas<T>()))
+__global__ void __launch_bounds__(T, (tile_ctas<M, BF16, T>()))
     sync_tile_kernel(const __grid_constant__ SyncArgs a) {
     constexpr int W = T / 32;
     constexpr int B = 4 * T;  // elements per block
@@ -394,7 +402,15 @@ cudaError_t tile_dispatch(const SyncArgs &a, int sm_count, int max_grid, cudaStr
         case 5: return tile_launch<5, BF16>(a, sm_count, max_grid, stream, grid_out);
         case 6: return tile_launch<6, BF16>(a, sm_count, max_grid, stream, grid_out);
         case 7: return tile_launch<7, BF16>(a, sm_count, max_grid, stream, grid_out);
-        default: return tile_launch<8, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 8: return tile_launch<8, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 9: return tile_launch<9, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 10: return tile_launch<10, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 11: return tile_launch<11, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 12: return tile_launch<12, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 13: return tile_launch<13, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 14: return tile_launch<14, BF16>(a, sm_count, max_grid, stream, grid_out);
+        case 15: return tile_launch<15, BF16>(a, sm_count, max_grid, stream, grid_out);
+        default: return tile_launch<16, BF16>(a, sm_count, max_grid, stream, grid_out);
     }
 }
 
