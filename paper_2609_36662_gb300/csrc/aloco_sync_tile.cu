@@ -112,9 +112,9 @@ __host__ __device__ constexpr int tile_threads() {
 }
 template <int M, bool BF16, int T>
 __host__ __device__ constexpr int tile_stages() {
-    return ALOCO_TILE_NS ? ALOCO_TILE_NS
-           : (BF16 || M > 8) ? 1
-           : (tile_fit<M, BF16, T, 2, false>() ? 2 : 1);
+    if (ALOCO_TILE_NS == 1) return 1;
+    const bool two = ALOCO_TILE_NS == 2 || (!BF16 && M <= 8);
+    return two && tile_fit<M, BF16, T, 2, false>() ? 2 : 1;
 }
 template <int M, bool BF16, int T, int NS>
 __host__ __device__ constexpr bool tile_gv() {
