@@ -34,7 +34,8 @@
 // Shared memory per CTA: the input buffer, 4096 x (8 + M x element size)
 // bytes, and the output tiles, 4096 x element size (plus 4096 x 8 for the
 // fp32 theta' and v' tiles where they fit; elsewhere threads store theta'
-// and v' themselves).  Worker counts beyond 8 use the split form.
+// and v' themselves).  It holds M <= 8 fp32 or M <= 16 bf16 replicas;
+// larger worker counts use the split form.
 //
 // A bounded wait that runs out (about 2 s) sets the round's error word; the
 // whole CTA leaves the block loop together at the next barrier, thread 0
@@ -49,7 +50,8 @@ namespace aloco {
 namespace {
 
 constexpr int kFlushBlocks = 8;
-constexpr int kFusedMax = 8;
+constexpr int kFusedMaxF32 = 8;   // fp32: the staging of M <= 8 replicas fits
+constexpr int kFusedMaxBF16 = 16; // bf16: M <= 16 (one CTA per SM above 8)
 
 // Shared memory of one SM and the largest a CTA may take (bytes), and the
 // part of each CTA's share the system reserves.
@@ -70,29 +72,30 @@ template <int M, int T>
 __host__ __device__ constexpr size_t static_bytes() {
     return (size_t)(T / 32) * (4 * M + 4 + 8 * M + 8 * (M + 1)) + 4096;
 }
-template <int T>
+// shared memory one of C CTAs per SM may take
+template <int C>
 __host__ __device__ constexpr size_t cta_budget() {
-    return T == 512 ? kSmemPerSm / 2 - kSmemReserved : kSmemPerCta;
+    return C == 1 ? kSmemPerCta : kSmemPerSm / C - kSmemReserved;
 }
 // The fp32 theta' and v' tiles fit beside the input and the replica tile.
-template <int M, bool BF16, int T>
+template <int M, bool BF16, int T, int C>
 __host__ __device__ constexpr bool tile_gv() {
     return in_bytes<M, BF16>() + (size_t)kI8Block * (esize<BF16>() + (BF16 ? 8 : 4)) +
                static_bytes<M, T>() <=
-           cta_budget<T>();
+           cta_budget<C>();
 }
-template <int M, bool BF16, int T>
+template <int M, bool BF16, int T, int C>
 __host__ __device__ constexpr size_t out_bytes() {
-    return tile_gv<M, BF16, T>() ? (size_t)kI8Block * (esize<BF16>() + (BF16 ? 8 : 4))
-                                 : (size_t)kI8Block * esize<BF16>();
+    return tile_gv<M, BF16, T, C>() ? (size_t)kI8Block * (esize<BF16>() + (BF16 ? 8 : 4))
+                                    : (size_t)kI8Block * esize<BF16>();
 }
-template <int M, bool BF16, int T>
+template <int M, bool BF16, int T, int C>
 __host__ __device__ constexpr size_t fused_smem() {
-    return in_bytes<M, BF16>() + out_bytes<M, BF16, T>();
+    return in_bytes<M, BF16>() + out_bytes<M, BF16, T, C>();
 }
-template <int M, bool BF16, int T>
+template <int M, bool BF16, int T, int C>
 __host__ __device__ constexpr bool fits() {
-    return fused_smem<M, BF16, T>() + static_bytes<M, T>() <= cta_budget<T>();
+    return fused_smem<M, BF16, T, C>() + static_bytes<M, T>() <= cta_budget<C>();
 }
 
 // Threads per CTA (T) and elements per thread (4096 / T), measured on
@@ -102,17 +105,27 @@ __host__ __device__ constexpr bool fits() {
 //     block in flight leaves the SM idle while the next block's copies land;
 //   fp32: T = 512 0.88-0.93 for M <= 3, against 0.70-0.82 with 1024
 //     threads; from M = 4 two 512-thread CTAs no longer fit.
-// ALOCO_I8_FUSED_T = 512 or 1024 forces one shape (a tuning knob).
+// ALOCO_I8_FUSED_T = 512 or 1024 and ALOCO_I8_FUSED_CTAS = 1 or 2 force a
+// shape (tuning knobs).
 #ifndef ALOCO_I8_FUSED_T
 #define ALOCO_I8_FUSED_T 0
 #endif
+#ifndef ALOCO_I8_FUSED_CTAS
+#define ALOCO_I8_FUSED_CTAS 0
+#endif
 template <int M, bool BF16>
 constexpr int fused_threads() {
-    constexpr int want = ALOCO_I8_FUSED_T ? ALOCO_I8_FUSED_T : 512;
-    return (want == 512 && !fits<M, BF16, 512>()) ? 1024 : want;
+    if (ALOCO_I8_FUSED_T == 1024) return 1024;
+    if (ALOCO_I8_FUSED_T == 512 && ALOCO_I8_FUSED_CTAS == 1) return 512;
+    return fits<M, BF16, 512, 2>() ? 512 : 1024;
 }
-template <int T>
-__host__ __device__ constexpr int fused_min_ctas() { return T == 512 ? 2 : 1; }
+// CTAs per SM the shared memory is planned for (and the register budget:
+// 64 registers a thread for 1024 threads per SM, 128 for 512)
+template <int M, bool BF16, int T>
+__host__ __device__ constexpr int fused_ctas() {
+    if (ALOCO_I8_FUSED_CTAS) return ALOCO_I8_FUSED_CTAS;
+    return (T == 512 && fits<M, BF16, 512, 2>()) ? 2 : 1;
+}
 
 // A thread's replica values of workers m0 and m0 + 1 (when m0 + 1 < M),
 // widened exactly, as PER / 2 pairs each.  Worker m's slice starts at
@@ -168,14 +181,14 @@ __device__ __forceinline__ float block_amax(const float (&y)[PER], unsigned *red
 }  // namespace
 
 template <int M, bool BF16, int T>
-__global__ void __launch_bounds__(T, (fused_min_ctas<T>()))
+__global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     int8_fused_kernel(const __grid_constant__ SyncArgs a,
                       const __grid_constant__ Int8Parts P) {
     constexpr int PER = kI8Block / T;  // elements per thread
     constexpr int NP = PER / 2;        // pairs per thread
     constexpr int W = T / 32;          // warps
     constexpr int ES = esize<BF16>();
-    constexpr bool GV = tile_gv<M, BF16, T>();
+    constexpr bool GV = tile_gv<M, BF16, T, fused_ctas<M, BF16, T>()>();
     constexpr uint32_t kGVBytes = kI8Block * 4;  // one fp32 array of a block
     constexpr uint32_t kXBytes = kI8Block * ES;  // one replica slice
     // Single buffers suffice: red_w is read between the block's two
@@ -530,8 +543,9 @@ template <int M, bool BF16>
 cudaError_t fused_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
                          int max_grid, cudaStream_t stream, int *grid_out) {
     constexpr int T = fused_threads<M, BF16>();
-    static_assert(fits<M, BF16, T>(), "fused INT8 staging exceeds shared memory");
-    constexpr size_t smem = fused_smem<M, BF16, T>();
+    constexpr int C = fused_ctas<M, BF16, T>();
+    static_assert(fits<M, BF16, T, C>(), "fused INT8 staging exceeds shared memory");
+    constexpr size_t smem = fused_smem<M, BF16, T, C>();
     static PerDevice occ_cache;  // attribute set-up and occupancy, per device
     const int dev = PerDevice::device();
     int occ = occ_cache.get(dev);
@@ -567,15 +581,29 @@ cudaError_t fused_dispatch(const SyncArgs &a, const Int8Parts &P, int sm_count,
         case 5: return fused_launch<5, BF16>(a, P, sm_count, max_grid, stream, grid_out);
         case 6: return fused_launch<6, BF16>(a, P, sm_count, max_grid, stream, grid_out);
         case 7: return fused_launch<7, BF16>(a, P, sm_count, max_grid, stream, grid_out);
-        default: return fused_launch<8, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 8: return fused_launch<8, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        default: break;
     }
+    if constexpr (BF16) {
+        switch (a.M) {
+            case 9: return fused_launch<9, true>(a, P, sm_count, max_grid, stream, grid_out);
+            case 10: return fused_launch<10, true>(a, P, sm_count, max_grid, stream, grid_out);
+            case 11: return fused_launch<11, true>(a, P, sm_count, max_grid, stream, grid_out);
+            case 12: return fused_launch<12, true>(a, P, sm_count, max_grid, stream, grid_out);
+            case 13: return fused_launch<13, true>(a, P, sm_count, max_grid, stream, grid_out);
+            case 14: return fused_launch<14, true>(a, P, sm_count, max_grid, stream, grid_out);
+            case 15: return fused_launch<15, true>(a, P, sm_count, max_grid, stream, grid_out);
+            case 16: return fused_launch<16, true>(a, P, sm_count, max_grid, stream, grid_out);
+            default: break;
+        }
+    }
+    return cudaErrorInvalidValue;
 }
 
 }  // namespace
 
 bool int8_fused_fits(int M, aloco_dtype dtype) {
-    (void)dtype;
-    return M >= 1 && M <= kFusedMax;
+    return M >= 1 && M <= (dtype == ALOCO_BF16 ? kFusedMaxBF16 : kFusedMaxF32);
 }
 
 cudaError_t launch_int8_fused(const SyncArgs &a, const Int8Parts &P, aloco_dtype dtype,
