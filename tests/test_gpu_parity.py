@@ -123,6 +123,24 @@ def test_unaligned_buffers(dt, offset):
     compare_round(wN, st, orc, g, v, xs)
 
 
+@pytest.mark.parametrize("pass_", [A.PASS_TILE, A.PASS_BULK_COPY], ids=["tile", "bulk_copy"])
+def test_bulk_passes_fall_back_on_unaligned_buffers(pass_):
+    """The bulk-copy passes need 16-byte aligned buffers: asked for on a
+    misaligned one, the round runs the register pass and still matches the
+    oracle."""
+    N, M = 300_007, 4
+    w = W.small(N + 8, M, "f32", seed=21)
+    g0, v0, xs0 = gpu_inputs(w)
+    g, v = g0[1:1 + N], v0[:N]
+    xs = [x[:N] for x in xs0]
+    wN = W.small(N, M, "f32", seed=21)
+    orc = run_oracle_round(g, v, xs, wN, wN.start_step, wN.H_sel[0])
+    st = run_gpu_round(g, v, xs, wN, wN.start_step, wN.H_sel[0],
+                       opts=A.default_opts(pass_=pass_))
+    assert st["status"] == A.OK and st["pass_used"] == A.PASS_REGISTERS
+    compare_round(wN, st, orc, g, v, xs)
+
+
 @pytest.mark.parametrize("mode", [A.CORR_FULL, A.CORR_MOMENTUM_ONLY,
                                   A.CORR_NONE])
 @pytest.mark.parametrize("normalize", [0, 1])
