@@ -126,8 +126,8 @@ typedef enum {
  *              replicas again (any M <= 16);
  *   INT8_FUSED one kernel that stages each block of theta, v and the
  *              replicas in shared memory, reading every replica once
- *              (M <= 8 fp32 or M <= 16 bf16 replicas; ALOCO_ERR_ARG
- *              otherwise);
+ *              (any M <= 16; above 8 fp32 replicas it stages each
+ *              block's replicas in groups);
  *   AUTO       the form measured faster on GB300 for (M, dtype).
  * aloco_sync / aloco_sync_ex reject the INT8 values and aloco_sync_int8 the
  * REGISTERS / BULK_COPY / TILE values with ALOCO_ERR_ARG. */

@@ -516,7 +516,7 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
              : int8_pass)
         return fail(ALOCO_ERR_ARG, "pass %d does not apply to this round", o.pass);
     if (int8 && o.pass == ALOCO_PASS_INT8_FUSED && !aloco::int8_fused_fits(M, dtype))
-        return fail(ALOCO_ERR_ARG, "the fused INT8 round takes M <= 8 (fp32) or M <= 16 (bf16)");
+        return fail(ALOCO_ERR_ARG, "the fused INT8 round takes M <= 16");
     if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
     if (N > 0 && (!global || !momentum || !locals))
         return fail(ALOCO_ERR_ARG, "NULL buffer");

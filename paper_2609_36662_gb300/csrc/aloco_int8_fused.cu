@@ -50,8 +50,7 @@ namespace aloco {
 namespace {
 
 constexpr int kFlushBlocks = 8;
-constexpr int kFusedMaxF32 = 8;   // fp32: the staging of M <= 8 replicas fits
-constexpr int kFusedMaxBF16 = 16; // bf16: M <= 16 (one CTA per SM above 8)
+constexpr int kFusedMax = 16;
 
 // Shared memory of one SM and the largest a CTA may take (bytes), and the
 // part of each CTA's share the system reserves.
@@ -61,11 +60,30 @@ constexpr size_t kSmemReserved = 1024;
 
 template <bool BF16>
 __host__ __device__ constexpr int esize() { return BF16 ? 2 : 4; }
-// theta, v (fp32) and the M replica slices of one block
+// Workers whose replica slices are staged at a time (a group), at most
+// `cap` per group in groups of near-equal size.
+__host__ __device__ constexpr int balanced_group(int M, int cap) {
+    return (M + (M + cap - 1) / cap - 1) / ((M + cap - 1) / cap);
+}
+// All M for M <= 8.  Above, groups of 3 for fp32: two 512-thread CTAs per
+// SM then fit, and measured 0.84-0.94 of the copy peak for M = 9..16
+// against 0.54-0.60 for groups of 8 on one 1024-thread CTA (the split form:
+// 0.66-0.67).  ALOCO_I8_FUSED_G caps the group (a tuning knob).
+#ifndef ALOCO_I8_FUSED_G
+#define ALOCO_I8_FUSED_G 0
+#endif
+template <int M, bool BF16>
+__host__ __device__ constexpr int fused_group() {
+    if (ALOCO_I8_FUSED_G) return balanced_group(M, ALOCO_I8_FUSED_G);
+    if (M <= 8 || BF16) return M;
+    return balanced_group(M, 3);
+}
+// theta, v (fp32) and one group's replica slices of one block
 template <int M, bool BF16>
 __host__ __device__ constexpr size_t in_bytes() {
-    return (size_t)kI8Block * (8 + M * esize<BF16>());
+    return (size_t)kI8Block * (8 + fused_group<M, BF16>() * esize<BF16>());
 }
+
 // the static shared arrays of the kernel and of the final reduction (an
 // upper bound)
 template <int M, int T>
@@ -127,13 +145,14 @@ __host__ __device__ constexpr int fused_ctas() {
     return (T == 512 && fits<M, BF16, 512, 2>()) ? 2 : 1;
 }
 
-// A thread's replica values of workers m0 and m0 + 1 (when m0 + 1 < M),
+// A thread's replica values of staging slots m0 and m0 + 1 (when m0 + 1 <
+// lim, the slots in use),
 // widened exactly, as PER / 2 pairs each.  Worker m's slice starts at
 // m x 4096 x element size; thread t's chunks of 4 elements sit at 4t + c x 4T.
 template <int M, bool BF16, int T>
 __device__ __forceinline__ void staged_reps(const unsigned char *sx, int m0, int t,
                                             float2 (&a)[kI8Block / T / 2],
-                                            float2 (&b)[kI8Block / T / 2]) {
+                                            float2 (&b)[kI8Block / T / 2], int lim = M) {
     constexpr int PER = kI8Block / T;
     constexpr int ES = esize<BF16>();
     const unsigned char *p0 = sx + (size_t)m0 * kI8Block * ES + 4 * t * ES;
@@ -145,7 +164,7 @@ __device__ __forceinline__ void staged_reps(const unsigned char *sx, int m0, int
             const uint2 w = *reinterpret_cast<const uint2 *>(p0 + off);
             a[2 * c] = make_float2(bf16_lo(w.x), bf16_hi(w.x));
             a[2 * c + 1] = make_float2(bf16_lo(w.y), bf16_hi(w.y));
-            if (m0 + 1 < M) {
+            if (m0 + 1 < lim) {
                 const uint2 u = *reinterpret_cast<const uint2 *>(p1 + off);
                 b[2 * c] = make_float2(bf16_lo(u.x), bf16_hi(u.x));
                 b[2 * c + 1] = make_float2(bf16_lo(u.y), bf16_hi(u.y));
@@ -154,7 +173,7 @@ __device__ __forceinline__ void staged_reps(const unsigned char *sx, int m0, int
             const float4 q = *reinterpret_cast<const float4 *>(p0 + off);
             a[2 * c] = make_float2(q.x, q.y);
             a[2 * c + 1] = make_float2(q.z, q.w);
-            if (m0 + 1 < M) {
+            if (m0 + 1 < lim) {
                 const float4 r = *reinterpret_cast<const float4 *>(p1 + off);
                 b[2 * c] = make_float2(r.x, r.y);
                 b[2 * c + 1] = make_float2(r.z, r.w);
@@ -189,21 +208,25 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     constexpr int W = T / 32;          // warps
     constexpr int ES = esize<BF16>();
     constexpr bool GV = tile_gv<M, BF16, T, fused_ctas<M, BF16, T>()>();
+    constexpr int G = fused_group<M, BF16>();    // workers staged at a time
+    constexpr int NG = (M + G - 1) / G;          // groups per block
+    constexpr bool GROUPED = NG > 1;
+    constexpr int EA = GROUPED ? G : M;          // energy accumulators a thread
     constexpr uint32_t kGVBytes = kI8Block * 4;  // one fp32 array of a block
     constexpr uint32_t kXBytes = kI8Block * ES;  // one replica slice
-    // Single buffers suffice: red_w is read between the block's two
-    // barriers and rewritten only after the second; red1 is read after the
-    // second and rewritten only after the next block's first.
-    __shared__ unsigned red_w[M][W];                  // [worker][warp]: conflict-free reads
+    // Single buffers suffice: red_w is read between a group's first barrier
+    // and the next barrier, and rewritten only after it; red1 is read after
+    // barrier 2 and rewritten only after the next block's first barrier.
+    __shared__ unsigned red_w[G][W];                  // [worker][warp]: conflict-free reads
     __shared__ unsigned red1[W];
     __shared__ double e_w[W][M];
-    __shared__ __align__(16) float2 sr[W][M + (M & 1)];  // per warp: (scale, 1/scale)
+    __shared__ __align__(16) float2 sr[W][G + (G & 1)];  // per warp: (scale, 1/scale)
     __shared__ __align__(8) unsigned long long full_bar;
     extern __shared__ __align__(128) unsigned char smem[];
     float *sg = reinterpret_cast<float *>(smem);
     float *sv = sg + kI8Block;
     unsigned char *sx = smem + 2 * kGVBytes;
-    unsigned char *ox = sx + M * kXBytes;             // theta' in the replica type
+    unsigned char *ox = sx + G * kXBytes;             // theta' in the replica type
     float *og = BF16 ? reinterpret_cast<float *>(ox + kXBytes)  // theta' (fp32)
                      : reinterpret_cast<float *>(ox);
     float *ov = og + kI8Block;                         // v' (GV only)
@@ -216,19 +239,25 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
-    float e_acc[M];
+    // energies: all M workers' over up to 8 blocks, or, with groups, one
+    // group's over one block
+    float e_acc[EA];
 #pragma unroll
-    for (int m = 0; m < M; ++m) e_acc[m] = 0.f;
+    for (int m = 0; m < EA; ++m) e_acc[m] = 0.f;
     int since_flush = 0;
-    auto flush = [&]() {
+    auto flush_rows = [&](int m0, int n) {
 #pragma unroll
-        for (int m = 0; m < M; ++m) {
+        for (int m = 0; m < EA; ++m) {
+            if (m >= n) break;
             float e = e_acc[m];
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) e += __shfl_down_sync(0xffffffffu, e, off);
-            if (lane == 0) e_w[warp][m] += (double)e;
+            if (lane == 0) e_w[warp][m0 + m] += (double)e;
             e_acc[m] = 0.f;
         }
+    };
+    auto flush = [&]() {
+        flush_rows(0, EA);
         since_flush = 0;
     };
 
@@ -246,36 +275,48 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         return l == kI8Block && a.nvec > 0 && (s % 8) == 0;
     };
     bool in_flight = false;  // thread 0: bulk loads issued and not yet seen complete
-    // thread 0: the bulk copies of the block at s
-    auto stage_bulk = [&](int64_t kbi, int64_t s) {
-        if (a.test_stall_tile1 != 0 && kbi == a.test_stall_tile1 - 1)
+    // thread 0: the bulk copies of group q of the block at s (theta and v
+    // come with group 0)
+    auto stage_bulk = [&](int64_t kbi, int64_t s, int q) {
+        if (q == 0 && a.test_stall_tile1 != 0 && kbi == a.test_stall_tile1 - 1)
             return;  // testing only: this phase never completes
-        mbar_arrive_expect_tx(bar, 2 * kGVBytes + M * kXBytes);
-        bulk_load(smem_addr(sg), a.g + s, kGVBytes, bar);
-        bulk_load(smem_addr(sv), a.v + s, kGVBytes, bar);
+        const int m0 = q * G;
+        const int gq = M - m0 < G ? M - m0 : G;
+        mbar_arrive_expect_tx(bar, (q == 0 ? 2 * kGVBytes : 0) + gq * kXBytes);
+        if (q == 0) {
+            bulk_load(smem_addr(sg), a.g + s, kGVBytes, bar);
+            bulk_load(smem_addr(sv), a.v + s, kGVBytes, bar);
+        }
 #pragma unroll
-        for (int m = 0; m < M; ++m)
-            bulk_load(smem_addr(sx + m * kXBytes),
-                      reinterpret_cast<const unsigned char *>(a.x[m]) + s * ES, kXBytes, bar);
+        for (int m = 0; m < G; ++m)
+            if (m < gq)
+                bulk_load(smem_addr(sx + m * kXBytes),
+                          reinterpret_cast<const unsigned char *>(a.x[m0 + m]) + s * ES,
+                          kXBytes, bar);
         in_flight = true;
     };
-    // every thread: its own elements of a short or unaligned block
-    auto stage_own = [&](int64_t s, int l) {
+    // every thread: its own elements of group q of a short or unaligned block
+    auto stage_own = [&](int64_t s, int l, int q) {
+        const int m0 = q * G;
+        const int gq = M - m0 < G ? M - m0 : G;
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
             const int e = el(i);
             const bool in = e < l;
-            sg[e] = in ? a.g[s + e] : 0.f;
-            sv[e] = in ? a.v[s + e] : 0.f;
+            if (q == 0) {
+                sg[e] = in ? a.g[s + e] : 0.f;
+                sv[e] = in ? a.v[s + e] : 0.f;
+            }
 #pragma unroll
-            for (int m = 0; m < M; ++m) {
+            for (int m = 0; m < G; ++m) {
+                if (m >= gq) break;
                 if constexpr (BF16)
                     reinterpret_cast<uint16_t *>(sx + m * kXBytes)[e] =
-                        in ? reinterpret_cast<const uint16_t *>(a.x[m])[s + e]
+                        in ? reinterpret_cast<const uint16_t *>(a.x[m0 + m])[s + e]
                            : (uint16_t)0;
                 else
                     reinterpret_cast<float *>(sx + m * kXBytes)[e] =
-                        in ? reinterpret_cast<const float *>(a.x[m])[s + e] : 0.f;
+                        in ? reinterpret_cast<const float *>(a.x[m0 + m])[s + e] : 0.f;
             }
         }
         // a later bulk copy may overwrite these bytes
@@ -304,9 +345,9 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     if (kb < nblocks) {
         locate_block(P, kb, start, len);
         if (!bulk_block(start, len))
-            stage_own(start, len);
+            stage_own(start, len, 0);
         else if (t == 0)
-            stage_bulk(kb, start);
+            stage_bulk(kb, start, 0);
     }
     for (; kb < nblocks; kb += gridDim.x) {
         const bool full = len == kI8Block;
@@ -316,116 +357,260 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         int nlen = 0;
         if (nk < nblocks) locate_block(P, nk, nstart, nlen);
         const bool next_bulk = nk < nblocks && bulk_block(nstart, nlen);
-        bool timed_out = false;
-        if (bulk) {
-            timed_out = !mbar_wait(bar, phase, nullptr);
-            if (t == 0 && !timed_out) in_flight = false;
-            phase ^= 1;
-        }
-
         float g[PER];
-#pragma unroll
-        for (int c = 0; c < PER; c += 4) {
-            const float4 q = *reinterpret_cast<const float4 *>(sg + el(c));
-            g[c] = q.x; g[c + 1] = q.y; g[c + 2] = q.z; g[c + 3] = q.w;
-        }
-        float2 g2[NP];
-#pragma unroll
-        for (int j = 0; j < NP; ++j) g2[j] = make_float2(g[2 * j], g[2 * j + 1]);
+        float2 g2[NP];    // theta, as pairs
+        float2 sum2[NP];  // the workers' decoded sum
+        if constexpr (!GROUPED) {
+            bool timed_out = false;
+            if (bulk) {
+                timed_out = !mbar_wait(bar, phase, nullptr);
+                if (t == 0 && !timed_out) in_flight = false;
+                phase ^= 1;
+            }
 
-        // 2. block maxima and energies of every worker
-        auto worker_max = [&](int m, const float2 (&x)[NP]) {
-            float2 d[NP];
 #pragma unroll
-            for (int j = 0; j < NP; ++j) d[j] = sub2(g2[j], x[j]);
-            float mf = 0.f;
-            float2 e2 = __fmul2_rn(d[0], d[0]);
-#pragma unroll
-            for (int j = 0; j < NP; ++j) {
-                mf = fmaxf(mf, fmaxf(fabsf(d[j].x), fabsf(d[j].y)));
-                if (j > 0) e2 = __ffma2_rn(d[j], d[j], e2);
+            for (int c = 0; c < PER; c += 4) {
+                const float4 q = *reinterpret_cast<const float4 *>(sg + el(c));
+                g[c] = q.x; g[c + 1] = q.y; g[c + 2] = q.z; g[c + 3] = q.w;
             }
-            const float e = __fadd_rn(e2.x, e2.y);
-            unsigned mx = __float_as_uint(mf);
-            if (!isfinite(e)) {  // a NaN or infinity: take the maximum by the bits
-                mx = 0;
 #pragma unroll
-                for (int j = 0; j < NP; ++j)
-                    mx = max(mx, max(__float_as_uint(fabsf(d[j].x)),
-                                     __float_as_uint(fabsf(d[j].y))));
-            }
-            e_acc[m] += e;
-            mx = __reduce_max_sync(0xffffffffu, mx);
-            if (lane == 0) red_w[m][warp] = mx;
-        };
-#pragma unroll
-        for (int m = 0; m < M; m += 2) {
-            float2 xa[NP], xb[NP];
-            staged_reps<M, BF16, T>(sx, m, t, xa, xb);
-            worker_max(m, xa);
-            if (m + 1 < M) worker_max(m + 1, xb);
-        }
-        if (++since_flush == kFlushBlocks) flush();
-        // barrier 1; a wait that ran out in any thread stops the whole CTA
-        if (__syncthreads_or(timed_out)) {
-            failed = true;
-            break;
-        }
-        // every thread wrote its part of the previous block's tiles before
-        // the barrier
-        if (pend && t == 0) store_tiles(pstart);
-        pend = false;
-        {
-            // every warp folds the W warp maxima of each worker (lane w reads
-            // warp w's); lane m keeps worker m's and writes its scale and
-            // reciprocal to this warp's table
-            unsigned mine = 0;
-#pragma unroll
-            for (int m = 0; m < M; ++m) {
-                const unsigned w =
-                    __reduce_max_sync(0xffffffffu, lane < W ? red_w[m][lane] : 0u);
-                mine = lane == m ? w : mine;
-            }
-            if (lane < M) {
-                const float sc = codec_scale(__uint_as_float(mine));
-                sr[warp][lane] = make_float2(sc, __frcp_rn(sc));
-            }
-            __syncwarp();
-        }
+            for (int j = 0; j < NP; ++j) g2[j] = make_float2(g[2 * j], g[2 * j + 1]);
 
-        // 3. encode, decode and sum in worker order
-        float2 sum2[NP];
+            // 2. block maxima and energies of every worker
+            auto worker_max = [&](int m, const float2 (&x)[NP]) {
+                float2 d[NP];
 #pragma unroll
-        for (int j = 0; j < NP; ++j) sum2[j] = splat2(-0.f);
-        auto add_worker = [&](float2 scr, const float2 (&x)[NP]) {
-            const float s = scr.x, r = scr.y;
-            bool ok = true;
-            float2 n[NP];
-#pragma unroll
-            for (int j = 0; j < NP; ++j) n[j] = code2_fast(sub2(g2[j], x[j]), r, ok);
-            if (!ok) {
+                for (int j = 0; j < NP; ++j) d[j] = sub2(g2[j], x[j]);
+                float mf = 0.f;
+                float2 e2 = __fmul2_rn(d[0], d[0]);
 #pragma unroll
                 for (int j = 0; j < NP; ++j) {
-                    const float2 d = sub2(g2[j], x[j]);
-                    n[j] = make_float2(codec_code_f(d.x, s, r), codec_code_f(d.y, s, r));
+                    mf = fmaxf(mf, fmaxf(fabsf(d[j].x), fabsf(d[j].y)));
+                    if (j > 0) e2 = __ffma2_rn(d[j], d[j], e2);
+                }
+                const float e = __fadd_rn(e2.x, e2.y);
+                unsigned mx = __float_as_uint(mf);
+                if (!isfinite(e)) {  // a NaN or infinity: take the maximum by the bits
+                    mx = 0;
+#pragma unroll
+                    for (int j = 0; j < NP; ++j)
+                        mx = max(mx, max(__float_as_uint(fabsf(d[j].x)),
+                                         __float_as_uint(fabsf(d[j].y))));
+                }
+                e_acc[m] += e;
+                mx = __reduce_max_sync(0xffffffffu, mx);
+                if (lane == 0) red_w[m][warp] = mx;
+            };
+#pragma unroll
+            for (int m = 0; m < M; m += 2) {
+                float2 xa[NP], xb[NP];
+                staged_reps<M, BF16, T>(sx, m, t, xa, xb);
+                worker_max(m, xa);
+                if (m + 1 < M) worker_max(m + 1, xb);
+            }
+            if (++since_flush == kFlushBlocks) flush();
+            // barrier 1; a wait that ran out in any thread stops the whole CTA
+            if (__syncthreads_or(timed_out)) {
+                failed = true;
+                break;
+            }
+            // every thread wrote its part of the previous block's tiles before
+            // the barrier
+            if (pend && t == 0) store_tiles(pstart);
+            pend = false;
+            {
+                // every warp folds the W warp maxima of each worker (lane w reads
+                // warp w's); lane m keeps worker m's and writes its scale and
+                // reciprocal to this warp's table
+                unsigned mine = 0;
+#pragma unroll
+                for (int m = 0; m < M; ++m) {
+                    const unsigned w =
+                        __reduce_max_sync(0xffffffffu, lane < W ? red_w[m][lane] : 0u);
+                    mine = lane == m ? w : mine;
+                }
+                if (lane < M) {
+                    const float sc = codec_scale(__uint_as_float(mine));
+                    sr[warp][lane] = make_float2(sc, __frcp_rn(sc));
+                }
+                __syncwarp();
+            }
+
+            // 3. encode, decode and sum in worker order
+#pragma unroll
+            for (int j = 0; j < NP; ++j) sum2[j] = splat2(-0.f);
+            auto add_worker = [&](float2 scr, const float2 (&x)[NP]) {
+                const float s = scr.x, r = scr.y;
+                bool ok = true;
+                float2 n[NP];
+#pragma unroll
+                for (int j = 0; j < NP; ++j) n[j] = code2_fast(sub2(g2[j], x[j]), r, ok);
+                if (!ok) {
+#pragma unroll
+                    for (int j = 0; j < NP; ++j) {
+                        const float2 d = sub2(g2[j], x[j]);
+                        n[j] = make_float2(codec_code_f(d.x, s, r), codec_code_f(d.y, s, r));
+                    }
+                }
+                // paired products, scalar sums (see mul2_rn)
+#pragma unroll
+                for (int j = 0; j < NP; ++j) {
+                    const float2 q = mul2_rn(n[j], splat2(s));
+                    sum2[j] = make_float2(__fadd_rn(sum2[j].x, q.x), __fadd_rn(sum2[j].y, q.y));
+                }
+            };
+#pragma unroll
+            for (int m = 0; m < M; m += 2) {
+                const float4 scr = *reinterpret_cast<const float4 *>(&sr[warp][m]);
+                float2 xa[NP], xb[NP];
+                staged_reps<M, BF16, T>(sx, m, t, xa, xb);
+                add_worker(make_float2(scr.x, scr.y), xa);
+                if (m + 1 < M) add_worker(make_float2(scr.z, scr.w), xb);
+            }
+
+        } else {
+            bool stop = false;
+            // 2.-3. per group of workers (one group unless fp32 M > 8)
+#pragma unroll
+            for (int q = 0; q < NG; ++q) {
+                const int m0 = q * G;                      // first worker
+                const int GQ = M - m0 < G ? M - m0 : G;    // workers in the group
+                bool timed_out = false;
+                if (bulk) {
+                    timed_out = !mbar_wait(bar, phase, nullptr);
+                    if (t == 0 && !timed_out) in_flight = false;
+                    phase ^= 1;
+                }
+                if (q == 0) {
+#pragma unroll
+                    for (int c = 0; c < PER; c += 4) {
+                        const float4 v4 = *reinterpret_cast<const float4 *>(sg + el(c));
+                        g[c] = v4.x; g[c + 1] = v4.y; g[c + 2] = v4.z; g[c + 3] = v4.w;
+                    }
+#pragma unroll
+                    for (int j = 0; j < NP; ++j) g2[j] = make_float2(g[2 * j], g[2 * j + 1]);
+                }
+
+                // 2. block maxima and energies of the group's workers (slot m of
+                // the staging holds worker m0 + m)
+                auto worker_max = [&](int m, const float2 (&x)[NP]) {
+                    float2 d[NP];
+#pragma unroll
+                    for (int j = 0; j < NP; ++j) d[j] = sub2(g2[j], x[j]);
+                    float mf = 0.f;
+                    float2 e2 = __fmul2_rn(d[0], d[0]);
+#pragma unroll
+                    for (int j = 0; j < NP; ++j) {
+                        mf = fmaxf(mf, fmaxf(fabsf(d[j].x), fabsf(d[j].y)));
+                        if (j > 0) e2 = __ffma2_rn(d[j], d[j], e2);
+                    }
+                    const float e = __fadd_rn(e2.x, e2.y);
+                    unsigned mx = __float_as_uint(mf);
+                    if (!isfinite(e)) {  // a NaN or infinity: take the maximum by the bits
+                        mx = 0;
+#pragma unroll
+                        for (int j = 0; j < NP; ++j)
+                            mx = max(mx, max(__float_as_uint(fabsf(d[j].x)),
+                                             __float_as_uint(fabsf(d[j].y))));
+                    }
+                    e_acc[m] += e;
+                    mx = __reduce_max_sync(0xffffffffu, mx);
+                    if (lane == 0) red_w[m][warp] = mx;
+                };
+#pragma unroll
+                for (int m = 0; m < G; m += 2) {
+                    if (m >= GQ) break;
+                    float2 xa[NP], xb[NP];
+                    staged_reps<G, BF16, T>(sx, m, t, xa, xb, GQ);
+                    worker_max(m, xa);
+                    if (m + 1 < GQ) worker_max(m + 1, xb);
+                }
+                if constexpr (GROUPED)
+                    flush_rows(m0, GQ);
+                else if (++since_flush == kFlushBlocks)
+                    flush();
+                // barrier 1 (of the group); a wait that ran out in any thread
+                // stops the whole CTA
+                if (__syncthreads_or(timed_out)) {
+                    stop = true;
+                    break;
+                }
+                if (q == 0) {
+                    // every thread wrote its part of the previous block's tiles
+                    // before the barrier
+                    if (pend && t == 0) store_tiles(pstart);
+                    pend = false;
+                }
+                {
+                    // every warp folds the W warp maxima of each worker (lane w
+                    // reads warp w's); lane m keeps worker m's and writes its
+                    // scale and reciprocal to this warp's table
+                    unsigned mine = 0;
+#pragma unroll
+                    for (int m = 0; m < G; ++m) {
+                        if (m >= GQ) break;
+                        const unsigned w =
+                            __reduce_max_sync(0xffffffffu, lane < W ? red_w[m][lane] : 0u);
+                        mine = lane == m ? w : mine;
+                    }
+                    if (lane < GQ) {
+                        const float sc = codec_scale(__uint_as_float(mine));
+                        sr[warp][lane] = make_float2(sc, __frcp_rn(sc));
+                    }
+                    __syncwarp();
+                }
+
+                // 3. encode, decode and sum in worker order
+                if (q == 0) {
+#pragma unroll
+                    for (int j = 0; j < NP; ++j) sum2[j] = splat2(-0.f);
+                }
+                auto add_worker = [&](float2 scr, const float2 (&x)[NP]) {
+                    const float sc = scr.x, r = scr.y;
+                    bool ok = true;
+                    float2 n[NP];
+#pragma unroll
+                    for (int j = 0; j < NP; ++j) n[j] = code2_fast(sub2(g2[j], x[j]), r, ok);
+                    if (!ok) {
+#pragma unroll
+                        for (int j = 0; j < NP; ++j) {
+                            const float2 d = sub2(g2[j], x[j]);
+                            n[j] = make_float2(codec_code_f(d.x, sc, r), codec_code_f(d.y, sc, r));
+                        }
+                    }
+                    // paired products, scalar sums (see mul2_rn)
+#pragma unroll
+                    for (int j = 0; j < NP; ++j) {
+                        const float2 qq = mul2_rn(n[j], splat2(sc));
+                        sum2[j] = make_float2(__fadd_rn(sum2[j].x, qq.x), __fadd_rn(sum2[j].y, qq.y));
+                    }
+                };
+#pragma unroll
+                for (int m = 0; m < G; m += 2) {
+                    if (m >= GQ) break;
+                    const float4 scr = *reinterpret_cast<const float4 *>(&sr[warp][m]);
+                    float2 xa[NP], xb[NP];
+                    staged_reps<G, BF16, T>(sx, m, t, xa, xb, GQ);
+                    add_worker(make_float2(scr.x, scr.y), xa);
+                    if (m + 1 < GQ) add_worker(make_float2(scr.z, scr.w), xb);
+                }
+                if (q + 1 < NG) {
+                    // every thread has read this group's slots and scales: the
+                    // next group of the same block goes into them
+                    __syncthreads();
+                    if (bulk) {
+                        if (t == 0) stage_bulk(kb, start, q + 1);
+                    } else {
+                        stage_own(start, len, q + 1);
+                    }
                 }
             }
-            // paired products, scalar sums (see mul2_rn)
-#pragma unroll
-            for (int j = 0; j < NP; ++j) {
-                const float2 q = mul2_rn(n[j], splat2(s));
-                sum2[j] = make_float2(__fadd_rn(sum2[j].x, q.x), __fadd_rn(sum2[j].y, q.y));
+            if (stop) {
+                failed = true;
+                break;
             }
-        };
-#pragma unroll
-        for (int m = 0; m < M; m += 2) {
-            const float4 scr = *reinterpret_cast<const float4 *>(&sr[warp][m]);
-            float2 xa[NP], xb[NP];
-            staged_reps<M, BF16, T>(sx, m, t, xa, xb);
-            add_worker(make_float2(scr.x, scr.y), xa);
-            if (m + 1 < M) add_worker(make_float2(scr.z, scr.w), xb);
-        }
 
+        }
         // 4. the mean's codec
         float v[PER];
 #pragma unroll
@@ -451,7 +636,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         // every thread has read this block's staging: the next block's bulk
         // copies go into the same buffer while the rest of this block runs
         // (a short or unaligned next block is staged after the stores)
-        if (next_bulk && t == 0) stage_bulk(nk, nstart);
+        if (next_bulk && t == 0) stage_bulk(nk, nstart, 0);
         const float rs = __frcp_rn(s);
         float gp[PER], vp[PER];
 #pragma unroll
@@ -506,7 +691,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         }
         b64 += (double)b32;  // at most PER terms per thread and block
         b32 = 0.f;
-        if (nk < nblocks && !next_bulk) stage_own(nstart, nlen);
+        if (nk < nblocks && !next_bulk) stage_own(nstart, nlen, 0);
 
         start = nstart;
         len = nlen;
@@ -582,20 +767,15 @@ cudaError_t fused_dispatch(const SyncArgs &a, const Int8Parts &P, int sm_count,
         case 6: return fused_launch<6, BF16>(a, P, sm_count, max_grid, stream, grid_out);
         case 7: return fused_launch<7, BF16>(a, P, sm_count, max_grid, stream, grid_out);
         case 8: return fused_launch<8, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 9: return fused_launch<9, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 10: return fused_launch<10, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 11: return fused_launch<11, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 12: return fused_launch<12, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 13: return fused_launch<13, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 14: return fused_launch<14, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 15: return fused_launch<15, BF16>(a, P, sm_count, max_grid, stream, grid_out);
+        case 16: return fused_launch<16, BF16>(a, P, sm_count, max_grid, stream, grid_out);
         default: break;
-    }
-    if constexpr (BF16) {
-        switch (a.M) {
-            case 9: return fused_launch<9, true>(a, P, sm_count, max_grid, stream, grid_out);
-            case 10: return fused_launch<10, true>(a, P, sm_count, max_grid, stream, grid_out);
-            case 11: return fused_launch<11, true>(a, P, sm_count, max_grid, stream, grid_out);
-            case 12: return fused_launch<12, true>(a, P, sm_count, max_grid, stream, grid_out);
-            case 13: return fused_launch<13, true>(a, P, sm_count, max_grid, stream, grid_out);
-            case 14: return fused_launch<14, true>(a, P, sm_count, max_grid, stream, grid_out);
-            case 15: return fused_launch<15, true>(a, P, sm_count, max_grid, stream, grid_out);
-            case 16: return fused_launch<16, true>(a, P, sm_count, max_grid, stream, grid_out);
-            default: break;
-        }
     }
     return cudaErrorInvalidValue;
 }
@@ -603,7 +783,8 @@ cudaError_t fused_dispatch(const SyncArgs &a, const Int8Parts &P, int sm_count,
 }  // namespace
 
 bool int8_fused_fits(int M, aloco_dtype dtype) {
-    return M >= 1 && M <= (dtype == ALOCO_BF16 ? kFusedMaxBF16 : kFusedMaxF32);
+    (void)dtype;
+    return M >= 1 && M <= kFusedMax;
 }
 
 cudaError_t launch_int8_fused(const SyncArgs &a, const Int8Parts &P, aloco_dtype dtype,

@@ -247,11 +247,11 @@ def test_pass_values_are_checked_against_the_round(lib):
                                    ctypes.byref(st))
     for p in (A.PASS_REGISTERS, A.PASS_BULK_COPY, A.PASS_TILE):
         assert int8(2, A.F32, p) == A.ERR_ARG
-    assert int8(9, A.F32, A.PASS_INT8_FUSED) == A.ERR_ARG
-    assert "fused" in A.last_error()
-    # bf16 replicas fit the fused form up to M = 16, the INT8 round's limit
-    assert int8(16, A.BF16, A.PASS_INT8_FUSED) in (A.ERR_CUDA, A.ERR_ARG)
-    assert "fused" not in A.last_error()
+    # the fused form takes every worker count the INT8 round takes (M <= 16)
+    for dt in (A.F32, A.BF16):
+        assert int8(16, dt, A.PASS_INT8_FUSED) in (A.ERR_CUDA, A.ERR_ARG)
+        assert "fused" not in A.last_error()
+    assert int8(17, A.BF16, A.PASS_INT8_FUSED) == A.ERR_ARG
     # accepted combinations get past argument checks (no device here)
     assert int8(4, A.F32, A.PASS_INT8_FUSED) in (A.ERR_CUDA, A.ERR_ARG)
     assert "fused" not in A.last_error()

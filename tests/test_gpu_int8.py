@@ -94,7 +94,7 @@ def _compare(w, st, corr, orc, g, v, xs):
 
 
 def _fits_fused(dt, M):
-    return M <= (16 if dt == "bf16" else 8)
+    return M <= 16
 
 
 FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
@@ -106,7 +106,7 @@ FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
 @pytest.mark.parametrize("parts_name", ["one_part", "ragged", "llama_like"])
 def test_int8_round_matches_oracle(dt, M, parts_name, form):
     if form == "fused" and not _fits_fused(dt, M):
-        pytest.skip("the fused form holds M <= 8 fp32 replicas")
+        pytest.skip("the fused form holds M <= 16")
     parts = PARTS[parts_name]
     N = sum(parts) if parts else 5 * 4096 + 333
     w = W.small(N, M, dt, seed=40 + M)
@@ -124,7 +124,7 @@ def test_int8_round_matches_oracle(dt, M, parts_name, form):
 
 @pytest.mark.parametrize("dt,M", [("f32", 1), ("f32", 4), ("f32", 7), ("bf16", 2),
                                   ("bf16", 5), ("bf16", 8), ("bf16", 9), ("bf16", 12),
-                                  ("bf16", 16)])
+                                  ("bf16", 16), ("f32", 9), ("f32", 12), ("f32", 16)])
 def test_int8_forms_agree_bit_for_bit(dt, M):
     """The fused and the split form take the same decisions in the same
     arithmetic: theta', v' and the replicas are bit-identical; the
@@ -153,14 +153,14 @@ def test_int8_forms_agree_bit_for_bit(dt, M):
 
 
 def test_int8_auto_form():
-    """AUTO takes the fused form wherever it fits (M <= 8 fp32, M <= 16
-    bf16), the split form beyond."""
+    """AUTO takes the fused form at every worker count the INT8 round
+    takes (fp32 above 8 workers stages each block's replicas in groups)."""
     for dt, M, want in (("bf16", 8, A.PASS_INT8_FUSED),
                         ("bf16", 9, A.PASS_INT8_FUSED),
                         ("bf16", 16, A.PASS_INT8_FUSED),
                         ("f32", 8, A.PASS_INT8_FUSED),
-                        ("f32", 9, A.PASS_INT8_SPLIT),
-                        ("f32", 16, A.PASS_INT8_SPLIT)):
+                        ("f32", 9, A.PASS_INT8_FUSED),
+                        ("f32", 16, A.PASS_INT8_FUSED)):
         w = W.small(3 * 4096 + 5, M, dt, seed=3)
         g, v, xs = gpu_inputs(w)
         sa, _ = schedule_pair(w.schedule)
