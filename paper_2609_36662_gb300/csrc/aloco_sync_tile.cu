@@ -104,11 +104,16 @@ __host__ __device__ constexpr bool tile_fit() {
 //     two for bf16); fp32 0.99-1.00 for M = 12..16 against 0.95-0.97 for
 //     the register pass, bf16 0.96-0.97 for M = 9..12 against 0.955-0.963.
 template <int M, bool BF16>
+__host__ __device__ constexpr int tile_threads_table() {
+    return M > 8 ? 512 : !BF16 ? 1024 : (M <= 4 ? 256 : 512);
+}
+// a forced thread count applies where one stage of its blocks fits
+template <int M, bool BF16>
 __host__ __device__ constexpr int tile_threads() {
-    return ALOCO_TILE_T ? ALOCO_TILE_T
-           : M > 8      ? 512
-           : !BF16      ? 1024
-                        : (M <= 4 ? 256 : 512);
+    if constexpr (ALOCO_TILE_T != 0) {
+        if (tile_fit<M, BF16, ALOCO_TILE_T, 1, false>()) return ALOCO_TILE_T;
+    }
+    return tile_threads_table<M, BF16>();
 }
 template <int M, bool BF16, int T>
 __host__ __device__ constexpr int tile_stages() {
