@@ -115,7 +115,7 @@ def test_intervals_with_controller_match_the_oracle_chain():
         executed.append(h)
         assessed += d.assessment != A.ASSESS_NONE
         step, k, h = done, k + 1, d.H_step
-    # the controller left its warm-up and judged intervals on both sides
+    # the controller left its warm-up and assessed intervals on both sides
     assert sum(executed) == budget and assessed >= 5, (executed, assessed)
     print("executed horizons:", executed)
     # final global model after `budget` inner steps of fp32 storage
