@@ -340,3 +340,26 @@ def test_adamw_defaults_and_argument_errors(lib):
     assert lib.aloco_adamw_step_normed(None, None, None, None, 0, 1, A.F32, A.F32,
                                        ctypes.byref(A.adamw_cfg()), None, None,
                                        None) == A.ERR_ARG
+
+
+def test_binding_constants_match_the_header():
+    """Every enumerator the binding mirrors has the header's value."""
+    import re
+    header = open(os.path.join(ROOT, "include", "aloco.h")).read()
+    values = {name: int(val) for name, val in
+              re.findall(r"\b(ALOCO_[A-Z0-9_]+)\s*=\s*(-?\d+)", header)}
+    mirror = {
+        "ALOCO_F32": A.F32, "ALOCO_BF16": A.BF16,
+        "ALOCO_OK": A.OK, "ALOCO_ERR_ARG": A.ERR_ARG, "ALOCO_ERR_CUDA": A.ERR_CUDA,
+        "ALOCO_ERR_NONFINITE": A.ERR_NONFINITE, "ALOCO_ERR_ALIAS": A.ERR_ALIAS,
+        "ALOCO_ERR_NOMEM": A.ERR_NOMEM,
+        "ALOCO_PASS_AUTO": A.PASS_AUTO, "ALOCO_PASS_REGISTERS": A.PASS_REGISTERS,
+        "ALOCO_PASS_BULK_COPY": A.PASS_BULK_COPY, "ALOCO_PASS_INT8_SPLIT": A.PASS_INT8_SPLIT,
+        "ALOCO_PASS_INT8_FUSED": A.PASS_INT8_FUSED, "ALOCO_PASS_TILE": A.PASS_TILE,
+        "ALOCO_CORR_FULL": A.CORR_FULL, "ALOCO_CORR_MOMENTUM_ONLY": A.CORR_MOMENTUM_ONLY,
+        "ALOCO_CORR_NONE": A.CORR_NONE,
+        "ALOCO_SCHED_COSINE": A.SCHED_COSINE, "ALOCO_SCHED_CONSTANT": A.SCHED_CONSTANT,
+        "ALOCO_SCHED_LINEAR": A.SCHED_LINEAR,
+    }
+    for name, val in mirror.items():
+        assert values.get(name) == val, (name, values.get(name), val)
