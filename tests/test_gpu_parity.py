@@ -344,3 +344,24 @@ def test_tile_pass_equals_register_pass_bit_for_bit(M, dt):
     assert s1["mean_sq_norm"] == pytest.approx(s2["mean_sq_norm"], rel=RTOL_STAT)
     for m in range(M):
         assert s1["drift"][m] == pytest.approx(s2["drift"][m], rel=RTOL_STAT)
+
+
+def test_auto_pass_choice():
+    """AUTO runs the tile pass from 2^27 parameters for fp32 with M = 1 or
+    5..16 and for bf16 with M <= 12, and the register pass elsewhere (fp32
+    M = 2..4, bf16 M >= 13, smaller rounds).  The buffers are zeros: only
+    the choice is checked."""
+    big, small = (1 << 27) + 4096, (1 << 27) - 4096
+    sched = A.Schedule.make()
+    cases = [(big, 8, torch.float32, A.PASS_TILE), (big, 1, torch.float32, A.PASS_TILE),
+             (big, 3, torch.float32, A.PASS_REGISTERS), (big, 4, torch.bfloat16, A.PASS_TILE),
+             (big, 13, torch.bfloat16, A.PASS_REGISTERS), (small, 8, torch.float32, A.PASS_REGISTERS)]
+    for n, M, dt, want in cases:
+        g = torch.zeros(n, device="cuda")
+        v = torch.zeros(n, device="cuda")
+        xs = [torch.zeros(n, dtype=dt, device="cuda") for _ in range(M)]
+        st = A.sync(g, v, xs, H_sel=150, H_base=100, step=4000, schedule=sched,
+                    outer_lr=0.7, outer_beta=0.9)
+        assert st["status"] == A.OK and st["pass_used"] == want, (n, M, dt, st["pass_used"])
+        del g, v, xs
+        torch.cuda.empty_cache()
