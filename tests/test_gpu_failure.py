@@ -131,3 +131,37 @@ def test_stalled_tile_pass_block_is_reported_and_the_device_stays_usable():
     assert st1["pass_used"] == A.PASS_TILE
     assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
     assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))
+
+
+def test_stalled_int8_worker_group_block_is_reported_and_the_device_stays_usable():
+    """The fused INT8 round with worker groups (fp32, M > 8): a block whose
+    first group never arrives makes the round report the timeout; the next
+    round equals the split form bit for bit."""
+    w = W.small(1 << 22, 12, "f32", seed=6)
+    kw = _kw(w)
+    fused = lambda: A.default_opts(pass_=A.PASS_INT8_FUSED)
+    g, v, xs = gpu_inputs(w)
+    st = A.sync_int8(g, v, xs, opts=fused(), **kw)
+    assert st["status"] == A.OK and st["pass_used"] == A.PASS_INT8_FUSED
+    block = 2 * st["grid"] + 9                # the third block of CTA 9
+    assert block < w.numel // 4096
+
+    g, v, xs = gpu_inputs(w)
+    A.test_stall_tile(block)
+    t0 = time.time()
+    st = A.sync_int8(g, v, xs, opts=fused(), raise_on_error=False, **kw)
+    took = time.time() - t0
+    assert st["status"] == A.ERR_CUDA
+    assert "timed out" in A.last_error()
+    assert 1.0 < took < 60.0, took
+    torch.cuda.synchronize()
+
+    g1, v1, x1 = gpu_inputs(w)
+    g2, v2, x2 = gpu_inputs(w)
+    st1 = A.sync_int8(g1, v1, x1, opts=fused(), **kw)
+    st2 = A.sync_int8(g2, v2, x2, opts=A.default_opts(pass_=A.PASS_INT8_SPLIT), **kw)
+    assert st1["status"] == st2["status"] == A.OK
+    assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
+    assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))
+    for a_, b_ in zip(x1, x2):
+        assert torch.equal(a_.view(torch.int32), b_.view(torch.int32))
