@@ -4,16 +4,20 @@
 A step is one outer synchronisation round (Algorithm 1: pseudo-gradients,
 average, D_t / C_t, corrected Nesterov step, replica reset) over one batch
 of synthetic worker endpoints, called through the C ABI.  The default
-workload is the Llama-style 150M parameter set (12 layers, d 768, tied
-embeddings; N = 137,841,408) with 8 fp32 worker replicas and consecutive
-rounds whose horizons are drawn by seed from {50, 100, 150, 200, 300},
-momentum carried across rounds.
+workload is the largest parameter set that fits one GPU: the Llama-style 3B
+set (26 layers, d 3072, 8 KV heads, untied; N = 2,814,016,512) with 8 bf16
+worker replicas and fp32 global weights and momentum (67.5 GB resident),
+over consecutive rounds whose horizons rise from 100 to 400 steps along a
+40k-step cosine schedule, momentum carried across rounds.
 
 Between timed rounds the replicas are refilled with new endpoints (this
 stands in for the workers' inner loops and is not timed); each round is
 bracketed by CUDA events on the launch stream, and the whole loop by a
-barrier and device synchronisation.  Every round reads and writes
-11 GB, far more than the 129 MB L2, so no L2 flush is needed.
+barrier and device synchronisation.  The reported step time is the median
+over the timed rounds.  A round of the default workload reads and writes
+135 GB, far more than the 129 MB L2; rounds whose buffers are smaller than
+four times the L2 are preceded by an untimed write of a buffer twice the
+L2's size, so that no round starts with its inputs in L2.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the fp64 oracle on the host
@@ -66,7 +70,65 @@ def parse_flat(name: str):
 
 def default_workload_name():
     from paper_2609_36662_gb300 import workloads as W
-    return W.llama_150m().name
+    return W.llama_3b().name
+
+
+L2_FALLBACK_BYTES = 129 * 1024 * 1024
+
+
+def l2_bytes(device) -> int:
+    import torch
+    try:
+        n = int(torch.cuda.get_device_properties(device).L2_cache_size)
+        return n if n > 0 else L2_FALLBACK_BYTES
+    except Exception:
+        return L2_FALLBACK_BYTES
+
+
+def needs_l2_flush(footprint_bytes: int, l2: int) -> bool:
+    """Whether a round's buffers are small enough that part of them could
+    still sit in L2 from the previous round (then each timed round is
+    preceded by an untimed write of a buffer twice the L2's size)."""
+    return footprint_bytes < 4 * l2
+
+
+def host_memory():
+    """Physical and available host memory in bytes (None where unknown),
+    and the cgroup limit if one is set."""
+    out = {"host_ram_bytes": None, "mem_available_bytes": None,
+           "cgroup_limit_bytes": None}
+    try:
+        out["host_ram_bytes"] = os.sysconf("SC_PAGE_SIZE") * \
+            os.sysconf("SC_PHYS_PAGES")
+    except Exception:
+        pass
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    out["mem_available_bytes"] = int(line.split()[1]) * 1024
+    except Exception:
+        pass
+    for path in ("/sys/fs/cgroup/memory.max",
+                 "/sys/fs/cgroup/memory/memory.limit_in_bytes"):
+        try:
+            with open(path) as f:
+                txt = f.read().strip()
+            if txt.isdigit() and int(txt) < (1 << 60):
+                out["cgroup_limit_bytes"] = int(txt)
+            break
+        except Exception:
+            continue
+    return out
+
+
+def pinned_budget(mem) -> int:
+    """Pinned host bytes the e2e leg may take: half of what is available
+    (and of the cgroup limit), so the host keeps room for the rest."""
+    cands = [v for v in (mem.get("mem_available_bytes"),
+                         mem.get("cgroup_limit_bytes"),
+                         mem.get("host_ram_bytes")) if v]
+    return int(0.5 * min(cands)) if cands else 0
 
 
 def hbm_peak():
@@ -216,6 +278,22 @@ def reduce_max(value: float, world: int, device=None) -> float:
     return float(t.item())
 
 
+def gather_partials(blob: bytes, world: int, device=None):
+    """Every rank's partial-sums blob (aloco_partials_t bytes), in rank
+    order: an all-gather of one fixed-size byte string per rank over the
+    process group (identity for one rank)."""
+    if world <= 1:
+        return [bytes(blob)]
+    import torch
+    import torch.distributed as dist
+    t = torch.frombuffer(bytearray(blob), dtype=torch.uint8)
+    if device is not None:
+        t = t.to(device)
+    out = [torch.empty_like(t) for _ in range(world)]
+    dist.all_gather(out, t)
+    return [o.cpu().numpy().tobytes() for o in out]
+
+
 def job_value(units_per_rank: float, seconds_max: float, world: int) -> float:
     """Whole-job throughput: the units every rank processed over the slowest
     rank's time."""
@@ -350,24 +428,26 @@ def run_reference(args, w):
     world, rank, _ = dist_env()
     if rank != 0:
         return 0
-    g = W.make_global(w, "cpu")
-    v = W.make_momentum(w, "cpu")
     rounds = W.steps_of_rounds(w, args.warmup + args.steps)
     step0, h0 = rounds[0]
 
-    def endpoints(n_chunks):
+    def inputs(n_chunks):
+        # the first n_chunks generator chunks of theta, v and the endpoints
+        # (a prefix of the workload's own vectors)
         n = min(w.numel, n_chunks * W.CHUNK)
+        g = W.make_global(w, "cpu", upto=n)
+        v = W.make_momentum(w, "cpu", upto=n)
         xs = [torch.empty(n, dtype=W.replica_dtype(w)) for _ in range(w.M)]
-        W.fill_replicas(w, g[:n], xs, 0, 0, n_chunks)
-        return xs
+        W.fill_replicas(w, g, xs, 0, 0, W.n_chunks_upto(n))
+        return g, v, xs
 
     # calibrate on the first chunk, then draw only the chunks the sample needs
-    xs = endpoints(1)
+    g, v, xs = inputs(1)
     sample = calibrated_sample(w, g, v, xs, step0, h0, args.ref_step_seconds,
                                args.comm)
-    need = (sample + W.CHUNK - 1) // W.CHUNK
+    need = W.n_chunks_upto(sample)
     if need > 1:
-        xs = endpoints(need)
+        g, v, xs = inputs(need)
     cores = host_cores()
     times = []
     for k, (step, hsel) in enumerate(rounds):
@@ -375,14 +455,15 @@ def run_reference(args, w):
                              threads=cores)
         if k >= args.warmup:
             times.append(t)
-    sec_per_round = statistics.mean(times) * w.numel / sample
+    sec_per_round = statistics.median(times) * w.numel / sample
     value = 1.0 / sec_per_round
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": sec_per_round * 1e3, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic",
+        "ms_per_step": sec_per_round * 1e3, "ms_per_step_stat": "median",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64",
+        "replica_dtype": w.dtype, "data": "synthetic",
         "config": dict(config_block(w), comm=args.comm),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores,
                          "kind": "oracle",
@@ -397,6 +478,21 @@ def run_reference(args, w):
     return 0
 
 
+def footprint_bytes(w) -> int:
+    """Bytes of the buffers one round reads (each is also written)."""
+    return w.bytes_per_round() // 2
+
+
+def l2_note(w, l2: int = L2_FALLBACK_BYTES) -> str:
+    if needs_l2_flush(footprint_bytes(w), l2):
+        return (f"L2 flushed before each timed round: the round's buffers "
+                f"({footprint_bytes(w) / 1e6:.0f} MB) are smaller than four "
+                f"times the L2, so an untimed write of {2 * l2 / 1e6:.0f} MB "
+                f"precedes each round")
+    return (f"no flush: each round moves {w.bytes_per_round() / 1e9:.1f} GB "
+            f"> 129 MB L2")
+
+
 def config_block(w):
     from paper_2609_36662_gb300 import workloads as W
     return {"workload": w.name, "N": w.numel, "M": w.M,
@@ -407,8 +503,7 @@ def config_block(w):
                        "ffn": w.shape.ffn, "vocab": w.shape.vocab,
                        "tied": w.shape.tied}),
             "bytes_per_round": w.bytes_per_round(),
-            "l2": f"no flush: each round moves {w.bytes_per_round() / 1e9:.1f} GB "
-                  "> 129 MB L2",
+            "l2": l2_note(w),
             "H_base": w.H_base, "start_step": w.start_step,
             "parallelism": "replicas only"}
 
@@ -462,11 +557,19 @@ def run_cuda(args, w):
     ev = [(torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in rounds]
 
+    l2 = l2_bytes(device)
+    flush_buf = None
+    if needs_l2_flush(footprint_bytes(w), l2):
+        flush_buf = torch.empty(2 * l2 // 4, dtype=torch.float32, device=device)
+
     def one_round(k):
         step, hsel = rounds[k]
         if k > 0:
             with torch.cuda.stream(stream):
                 W.fill_replicas(w, g, xs, k)      # untimed: the inner loops
+        if flush_buf is not None:
+            with torch.cuda.stream(stream):
+                flush_buf.fill_(float(k))         # untimed: evict the L2
         ev[k][0].record(stream)
         if args.comm == "int8":
             st = A.sync_int8(g, v, xs, parts=parts, H_sel=hsel,
@@ -505,9 +608,10 @@ def run_cuda(args, w):
     kernel_name = {2: "sync_tma_kernel", 3: "int8_split_kernels",
                    4: "int8_fused_kernel", 5: "sync_tile_kernel"}.get(st_first.get("pass_used"),
                                                "sync_kernel")
-    ms_step = statistics.mean(step_ms)
-    ms_step = reduce_max(ms_step, world, device)
-    ms_kern = reduce_max(statistics.mean(kern_ms), world, device)
+    # median over the timed rounds (each rank), then the slowest rank
+    ms_step_mean = reduce_max(statistics.mean(step_ms), world, device)
+    ms_step = reduce_max(statistics.median(step_ms), world, device)
+    ms_kern = reduce_max(statistics.median(kern_ms), world, device)
     value = job_value(1.0, ms_step / 1e3, world)
     peak, peak_kind = hbm_peak()
     achieved = w.bytes_per_round() / (ms_kern / 1e3) / 1e9
@@ -523,14 +627,18 @@ def run_cuda(args, w):
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": ms_step, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "ms_per_step": ms_step, "ms_per_step_stat": "median",
+            "ms_per_step_mean": ms_step_mean, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None,
+            # arithmetic type of the path; the replicas are stored as below
+            "dtype": "f32", "replica_dtype": w.dtype,
             "data": "synthetic (seeded; Llama-shaped parameter set, "
                     "shared/private drift noise)",
-            "config": dict(config_block(w), comm=args.comm),
+            "config": dict(config_block(w), comm=args.comm,
+                           l2=l2_note(w, l2)),
             "rounds_per_s_per_gpu": 1e3 / ms_step,
             "elem_per_s": value * w.numel * w.M,
-            "kernel_ms": ms_kern,
+            "kernel_ms": ms_kern, "kernel_ms_stat": "median",
             "hbm_gbs": achieved,
             "frac_of_nominal_8000": achieved / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
@@ -568,25 +676,31 @@ def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
     rbytes = w.replica_bytes()
     h2d = w.numel * (8 + w.M * rbytes)
     d2h = w.numel * 8
-    try:
-        page = os.sysconf("SC_PAGE_SIZE") * os.sysconf("SC_PHYS_PAGES")
-    except Exception:
-        page = 0
-    if page and (h2d + d2h) > 0.4 * page:
+    # pinned host state: theta, v and the endpoints (theta', v' come back
+    # into theta, v); the INT8 leg copies theta', v' out to two more arrays
+    pinned = h2d + (d2h if int8_parts is not None else 0)
+    mem = host_memory()
+    budget = pinned_budget(mem)
+    if budget and pinned > budget:
         return {"value": None, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h,
-                "skipped": "pinned host buffers would exceed 40% of host RAM"}
+                "d2h_bytes_per_step": d2h, "pinned_bytes": pinned, **mem,
+                "skipped": f"the pinned host state ({pinned / 1e9:.1f} GB) "
+                           f"exceeds half of the host memory available "
+                           f"({budget / 1e9:.1f} GB allowed)"}
+    t_pin = time.perf_counter()
     hg = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
     hv = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
     hx = [torch.empty(w.numel, dtype=W.replica_dtype(w), pin_memory=True)
           for _ in range(w.M)]
+    if int8_parts is not None:
+        og = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
+        ov = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
+    t_pin = time.perf_counter() - t_pin
     W.fill_replicas(w, g, xs, 0)
     hg.copy_(g)
     hv.copy_(v)
     for a, b in zip(hx, xs):
         a.copy_(b)
-    og = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
-    ov = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
     ms = []
     n_total = args.e2e_warmup + args.e2e_steps
     for k in range(n_total):
@@ -616,13 +730,140 @@ def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
         e1.synchronize()
         if k >= args.e2e_warmup:
             ms.append(e0.elapsed_time(e1))
-    m = reduce_max(statistics.mean(ms), world, device)
-    return {"value": job_value(1.0, m / 1e3, world), "unit": UNIT,
-            "ms_per_step": m, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h + 8 * (w.M + 2),
-            "steps": args.e2e_steps,
-            "api": "aloco_sync_host" if int8_parts is None else
-                   "copies + aloco_sync_int8"}
+    m = reduce_max(statistics.median(ms), world, device)
+    out = {"value": job_value(1.0, m / 1e3, world), "unit": UNIT,
+           "ms_per_step": m, "ms_per_step_stat": "median",
+           "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h + 8 * (w.M + 2),
+           "steps": args.e2e_steps,
+           "api": "aloco_sync_host" if int8_parts is None else
+                  "copies + aloco_sync_int8",
+           "pinned_bytes": pinned, "pin_alloc_s": t_pin,
+           "host_ram_bytes": mem["host_ram_bytes"]}
+    del hg, hv, hx
+    return out
+
+
+# ----------------------------------------------------------- sharded mode
+
+def run_shard(args, w):
+    """The round over a vector cut into contiguous shards at generator-chunk
+    boundaries (aloco_sync_shard on each, aloco_combine_partials in shard
+    order).  One process: --shards G shards run one after another on the one
+    GPU.  Under torchrun: rank r holds and runs shard r of WORLD_SIZE shards,
+    and the ranks all-gather their partials (one small struct each) over
+    NCCL before combining them, so every rank obtains the same D_t and C_t.
+    A step is one whole round (every shard, the exchange and the combine),
+    timed on the host around calls that return once their kernels are done;
+    the value is whole rounds per second (total work fixed as ranks are
+    added: strong scaling)."""
+    import torch
+    from paper_2609_36662_gb300 import aloco as A
+    from paper_2609_36662_gb300 import workloads as W
+
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", torch.cuda.current_device())
+    A.load()
+    G = world if world > 1 else max(1, args.shards)
+    mine = [rank] if world > 1 else list(range(G))
+    rounds = W.steps_of_rounds(w, args.warmup + args.steps)
+    pieces = []
+    for k in mine:
+        c_lo, c_hi = W.shard_chunks(w, G, k)
+        g = W.make_global(w, device, chunks=(c_lo, c_hi))
+        v = torch.zeros_like(g)
+        xs = [torch.empty(g.numel(), dtype=W.replica_dtype(w), device=device)
+              for _ in range(w.M)]
+        W.fill_replicas(w, g, xs, 0, c_lo, c_hi)
+        pieces.append((c_lo, c_hi, g, v, xs))
+    s = w.schedule
+    sched = A.Schedule.make(s.kind, s.peak_lr, s.final_lr, s.warmup_steps,
+                            s.total_steps)
+    stream = torch.cuda.Stream(device)
+    opts = A.default_opts(time_kernel=1, pass_=PASSES[args.pass_])
+    step_ms, kern_ms, statuses, D, C = [], [], [], [], []
+
+    def one_round(k):
+        step, hsel = rounds[k]
+        if k > 0:
+            with torch.cuda.stream(stream):
+                for c_lo, c_hi, g, v, xs in pieces:
+                    W.fill_replicas(w, g, xs, k, c_lo, c_hi)   # untimed
+        stream.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        t0 = time.perf_counter()
+        blobs, ms = [], 0.0
+        for _, _, g, v, xs in pieces:
+            rc, part = A.sync_shard(g, v, xs, H_sel=hsel, H_base=w.H_base,
+                                    step=step, schedule=sched,
+                                    outer_lr=w.outer_lr,
+                                    outer_beta=w.outer_beta, opts=opts,
+                                    stream=stream)
+            blobs.append(part.to_bytes())
+            ms += max(part.kernel_ms, 0.0)
+        if world > 1:
+            blobs = gather_partials(blobs[0], world, device)
+        st = A.combine_partials([A.Partials.from_bytes(b) for b in blobs])
+        t1 = time.perf_counter()
+        return (t1 - t0) * 1e3, ms, st
+
+    for k in range(args.warmup):
+        one_round(k)
+    torch.cuda.synchronize()
+    with ClockSampler(device.index) as clocks:
+        for k in range(args.warmup, args.warmup + args.steps):
+            t, ms, st = one_round(k)
+            step_ms.append(t)
+            kern_ms.append(ms)
+            statuses.append(st["status"])
+            D.append(st["D"])
+            C.append(st["C"])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    ms_step = reduce_max(statistics.median(step_ms), world, device)
+    ms_kern = reduce_max(statistics.median(kern_ms), world, device)
+    peak, peak_kind = hbm_peak()
+    # bytes this rank's shards move in one round, over their kernel time
+    my_bytes = sum(g.numel() for _, _, g, _, _ in pieces) * \
+        (2 * (8 + w.M * w.replica_bytes()))
+    achieved = my_bytes / (ms_kern / 1e3) / 1e9 if ms_kern > 0 else None
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": 1e3 / ms_step, "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms_step, "ms_per_step_stat": "median",
+            "higher_is_better": True, "scaling": "strong",
+            "vs_baseline": None, "dtype": "f32", "replica_dtype": w.dtype,
+            "data": "synthetic (seeded; Llama-shaped parameter set, "
+                    "shared/private drift noise)",
+            "config": dict(config_block(w), comm="fp32",
+                           parallelism=(f"shard{G}" if world > 1 else
+                                        f"{G} shards in sequence on one GPU"),
+                           shard_elems=[g.numel() for _, _, g, _, _ in pieces]
+                           if world == 1 else None),
+            "kernel_ms": ms_kern, "kernel_ms_stat": "median",
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
+                         "unit": "GB/s",
+                         "frac": achieved / peak if achieved else None,
+                         "peak_source": peak_kind, "traffic": None,
+                         "kernel": "shard kernels (rank 0)",
+                         "algorithmic_bytes_per_launch": my_bytes},
+            "cpu_baseline": None, "e2e": None,
+            "gpu_launches": args.steps * len(pieces),
+            "clocks": clocks.summary(),
+            "status_ok": all(x == A.OK for x in statuses),
+            "D_last": D[-1], "C_last": C[-1],
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
 
 
 # ------------------------------------------------------ inner AdamW mode
@@ -725,13 +966,14 @@ def run_adamw_reference(args, w):
         t, n = adamw_oracle_sample(small, xs, gs, m1, m2, sample, threads=cores)
         if k >= args.warmup:
             times.append(t)
-    sec = statistics.mean(times) * w.numel / sample
+    sec = statistics.median(times) * w.numel / sample
     value = 1.0 / sec
     line = {"impl": "reference", "metric": ADAMW_METRIC, "value": value,
             "unit": ADAMW_UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": sec * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f64", "data": "synthetic", "config": adamw_config(w),
+            "dtype": "f64", "replica_dtype": w.dtype, "data": "synthetic",
+            "config": adamw_config(w),
             "cpu_baseline": {"value": value, "unit": ADAMW_UNIT, "cores": cores,
                              "kind": "oracle",
                              "sample": f"first {sample} elements of each of "
@@ -804,8 +1046,8 @@ def run_adamw(args, w):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    ms = statistics.mean(ev[k][0].elapsed_time(ev[k][1])
-                         for k in range(args.warmup, args.warmup + args.steps))
+    ms = statistics.median(ev[k][0].elapsed_time(ev[k][1])
+                           for k in range(args.warmup, args.warmup + args.steps))
     ms = reduce_max(ms, world, device)
     st = A.adamw_step(xs, gs, m1, m2, A.adamw_cfg(lr=ADAMW_LR, step=ADAMW_STEP0),
                       opts=opts, stream=stream)
@@ -835,7 +1077,7 @@ def run_adamw(args, w):
             e1.synchronize()
             if k >= args.e2e_warmup:
                 times.append(e0.elapsed_time(e1))
-        m_e = reduce_max(statistics.mean(times), world, device)
+        m_e = reduce_max(statistics.median(times), world, device)
         e2e = {"value": job_value(1.0, m_e / 1e3, world), "unit": ADAMW_UNIT,
                "ms_per_step": m_e,
                "h2d_bytes_per_step": sum(g.numel() * g.element_size() for g in gs),
@@ -844,8 +1086,9 @@ def run_adamw(args, w):
         line = {
             "metric": ADAMW_METRIC, "value": value, "unit": ADAMW_UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f32",
+            "ms_per_step": ms, "ms_per_step_stat": "median",
+            "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "replica_dtype": w.dtype,
             "data": "synthetic (seeded replicas, gradients and moments)",
             "config": adamw_config(w),
             "elem_per_s": value * w.numel * w.M,
@@ -937,6 +1180,7 @@ def run_interval(args, w):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": tot_ms / len(hs), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "replica_dtype": w.dtype,
             "data": "synthetic (seeded replicas, fixed synthetic gradients)",
             "config": dict(adamw_config(w), mode="interval",
                            controller="C4 recipe: H_base 500 in [250, 750], "
@@ -959,8 +1203,8 @@ def main(argv=None):
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
     p.add_argument("--workload", default=None,
-                   help="workload name (default: the Llama-style 150M set, "
-                        "8 fp32 workers)")
+                   help="workload name (default: the Llama-style 3B set, "
+                        "8 bf16 workers)")
     p.add_argument("--cpu-seconds", type=float, default=10.0)
     p.add_argument("--ref-step-seconds", type=float, default=3.0)
     p.add_argument("--e2e-steps", type=int, default=5)
@@ -980,6 +1224,10 @@ def main(argv=None):
                    default="computed",
                    help="--mode adamw: compute the clipping norms (two "
                         "passes) or take them from the caller (one pass)")
+    p.add_argument("--shards", type=int, default=0,
+                   help="run the round as shards (aloco_sync_shard + "
+                        "aloco_combine_partials): G shards in sequence on "
+                        "one GPU, or one shard per rank under torchrun")
     p.add_argument("--list", action="store_true")
     args = p.parse_args(argv)
     table = workloads_by_name()
@@ -1006,6 +1254,8 @@ def main(argv=None):
         return run_interval(args, w)
     if args.impl == "reference":
         return run_reference(args, w)
+    if args.shards > 0:
+        return run_shard(args, w)
     return run_cuda(args, w)
 
 

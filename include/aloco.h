@@ -119,8 +119,8 @@ typedef enum {
  *              replica reset as M bulk copies of it (M <= 16, 16-byte
  *              aligned buffers, N >= 4096; otherwise REGISTERS runs);
  *   AUTO       the fastest as measured on GB300 for (M, dtype, N): TILE
- *              from 2^27 parameters for bf16 replicas and for fp32 with
- *              M = 1 or 5..8, else REGISTERS.
+ *              from 2^27 parameters for bf16 replicas with M <= 12 and for
+ *              fp32 with M = 1 or 5..16, else REGISTERS.
  * The INT8-communicated round (aloco_sync_int8) has two forms of its own:
  *   INT8_SPLIT a block-scale kernel, then an apply kernel that reads the
  *              replicas again (any M <= 16);
@@ -140,11 +140,27 @@ typedef enum {
     ALOCO_PASS_TILE = 5
 } aloco_pass;
 
+/* How a round call waits for its kernel (aloco_sync_ex, aloco_sync_int8 and
+ * the shard calls):
+ *   SPIN   the calling thread polls the device-mapped page that the round's
+ *          last block publishes its statistics to, checking the stream every
+ *          few hundred reads.  Lowest latency (the call returns a few
+ *          microseconds after the last block), but the thread keeps one host
+ *          core busy for the whole round, including any time the stream is
+ *          queued behind earlier work.
+ *   BLOCK  the call records a blocking-sync CUDA event behind the kernel and
+ *          waits on it: the thread sleeps until the round has completed, then
+ *          reads the same published statistics.  For callers that run the
+ *          round on a busy stream or need the core; each call pays the
+ *          event's wake-up latency.
+ * Outputs and statistics are the same in both modes. */
+typedef enum { ALOCO_WAIT_SPIN = 0, ALOCO_WAIT_BLOCK = 1 } aloco_wait;
+
 /* Options.  aloco_default_opts() fills the paper's settings
  * (Tab. AutoLoCo configuration): mu_min 0.45, mu_max 0.90, kappa_max 1.6,
  * eps 1e-8, normalize off, FULL correction, no kernel timing, the tuned
- * launch configuration, default stream, AUTO pass.  Passing NULL where an opts pointer is accepted means these
- * defaults. */
+ * launch configuration, default stream, AUTO pass, SPIN wait.  Passing NULL
+ * where an opts pointer is accepted means these defaults. */
 typedef struct aloco_opts {
     double mu_min;
     double mu_max;
@@ -162,7 +178,7 @@ typedef struct aloco_opts {
                              statistics in their last bits.                  */
     void *stream;         /* cudaStream_t; NULL = legacy default stream      */
     int32_t pass;         /* aloco_pass: which fused kernel runs the round   */
-    int32_t reserved;
+    int32_t wait;         /* aloco_wait: how the host waits for the round    */
 } aloco_opts_t;
 
 /* Correction context of one interval (App. B.2, B.4). */
@@ -284,6 +300,85 @@ int aloco_sync_host(float *global, float *momentum, const void *const *locals,
                     const aloco_schedule_t *schedule, double outer_lr,
                     double outer_beta, size_t chunk_elems,
                     const aloco_opts_t *opts, aloco_stats_t *stats_out);
+
+/* ------------------------------------------------------------------------
+ * Sharded rounds (the synchronisation of Algorithm 1 over a parameter vector
+ * split into contiguous shards, for instance one shard per GPU).
+ *
+ * Every element of the round depends only on its own inputs and the round's
+ * scalars (rho, mu_t, eta_out come from the schedule, not from the data), so
+ * a shard can run the whole fused pass on its own range.  Only D_t and C_t
+ * (Eq. adaptive-h-core-diagnostics) are sums over the whole vector: each
+ * shard returns its partial sums, the shards' partials are exchanged (an
+ * all-gather of one small struct per shard), and every holder combines them
+ * in the same fixed shard order, so all of them obtain the same statistics.
+ * ---------------------------------------------------------------------- */
+
+/* Partial sums of one shard of a round, before combination. */
+typedef struct aloco_partials {
+    double drift[ALOCO_MAX_WORKERS];  /* sum over the shard of Delta_m^2      */
+    double sum_sq;                    /* sum over the shard of the squared
+                                         aggregate, in the pass's own units   */
+    double sq_scale;                  /* factor that turns the summed sum_sq
+                                         into ||Dbar||^2 (1/M^2 for the plain
+                                         round, which sums (sum_m Delta_m)^2;
+                                         1 for the INT8 round)                */
+    double eps;                       /* opts->eps of the shard               */
+    aloco_correction_t corr;          /* correction context applied           */
+    int64_t nonfinite;                /* elements whose theta' or v' is not
+                                         finite                               */
+    int64_t n;                        /* elements of the shard                */
+    int32_t M;
+    int32_t pass_used;                /* aloco_pass that ran (0: empty shard) */
+    float kernel_ms;                  /* fused-pass duration, or -1           */
+    int32_t reserved;
+} aloco_partials_t;
+
+/* One shard of an outer round: aloco_sync_ex on the n_shard elements that
+ * global, momentum and locals[m] point to (the shard's first element), but
+ * instead of the finished statistics it returns the shard's partial sums in
+ * *partials_out (required).  theta', v' and the replica reset of the shard are
+ * written in place and equal aloco_sync_ex's on the same elements bit for bit
+ * (the fused pass is elementwise); only the grouping of the partial sums
+ * differs from an unsharded round.  The kernel is chosen for the shard's size
+ * (see aloco_pass); shards whose pointers are 16-byte aligned keep the
+ * vector paths.  n_shard = 0 is allowed (no kernel runs; zero partials with
+ * the correction context).  Returns ALOCO_ERR_NONFINITE, with the partials
+ * filled, when the shard produced a non-finite theta' or v'.  Other
+ * arguments, errors and the wait as aloco_sync_ex. */
+int aloco_sync_shard(float *global, float *momentum, void *const *locals,
+                     size_t n_shard, int M, aloco_dtype dtype, int64_t H_sel,
+                     int64_t H_base, int64_t step,
+                     const aloco_schedule_t *schedule, double outer_lr,
+                     double outer_beta, const aloco_opts_t *opts,
+                     aloco_partials_t *partials_out);
+
+/* The INT8-communicated round (aloco_sync_int8) on one shard.  The shard's
+ * part_sizes describe the tensor parts it holds; codec blocks restart at
+ * every part, so a shard made of whole tensor parts encodes exactly the
+ * blocks the unsharded round would.  Partials as aloco_sync_shard. */
+int aloco_sync_int8_shard(float *global, float *momentum, void *const *locals,
+                          size_t n_shard, int M, aloco_dtype dtype,
+                          int64_t H_sel, int64_t H_base, int64_t step,
+                          const aloco_schedule_t *schedule, double outer_lr,
+                          double outer_beta, const int64_t *part_sizes,
+                          int n_parts, const aloco_opts_t *opts,
+                          aloco_partials_t *partials_out);
+
+/* Combine the partials of n_shards >= 1 shards of one round (host only, no
+ * GPU): the drift energies, the squared aggregate and the non-finite counts
+ * are added shard by shard in array order, then
+ *   D = (1/M) sum_m drift_m,  ||Dbar||^2 = sq_scale sum_sq,
+ *   C = M ||Dbar||^2 / (D + eps)          (Eq. adaptive-h-core-diagnostics).
+ * Every holder that combines the same partials in the same order obtains
+ * bit-identical statistics.  stats_out->grid is n_shards, kernel_ms the
+ * largest shard's time (or -1), pass_used the first non-empty shard's.
+ * ALOCO_ERR_ARG when the shards disagree on M, eps, sq_scale or the
+ * correction context (they are not shards of one round); ALOCO_ERR_NONFINITE,
+ * with the statistics filled, when any shard counted a non-finite element or
+ * D or C is not finite. */
+int aloco_combine_partials(const aloco_partials_t *shards, int n_shards,
+                           aloco_stats_t *stats_out);
 
 /* ------------------------------------------------------------------------
  * INT8 pseudo-gradient communication (App. G.1).
@@ -586,30 +681,36 @@ int aloco_ctrl_load(aloco_ctrl_state_t *state, const void *buf, size_t len);
  * that cudaMalloc / cudaFree imply.  aloco_sync_ex, by contrast, allocates a
  * cached per-device workspace on its first call.
  *
- * Arguments, results, status codes and numerics are those of aloco_sync_ex
- * (same kernel, same grid, same fixed-order reductions), except that
- * opts->time_kernel is ignored (stats_out->kernel_ms is -1).  The caller
- * still provides every input and output buffer.
+ * Arguments, results, status codes and numerics are those of aloco_sync_ex:
+ * the kernel is chosen by the same rule from opts->pass, M, dtype and N (the
+ * tile, bulk-copy or register pass; pass_used reports it) and launched with
+ * the same grid, so theta', v', the replicas and the fixed-order statistics
+ * equal aloco_sync_ex's bit for bit on the same inputs.  Exceptions:
+ * opts->time_kernel is ignored (stats_out->kernel_ms is -1), and the call
+ * cannot run under stream capture (it ends with a stream synchronisation;
+ * a call on a capturing stream returns ALOCO_ERR_ARG before enqueuing
+ * anything).  The caller still provides every input and output buffer.
  *
  * Scratch: the per-block partial sums live in one statically sized device
  * array inside the library (about 560 KB: ALOCO_NOALLOC_MAX_BLOCKS rows of
  * ALOCO_MAX_WORKERS + 1 doubles plus counters), which every GPU that loads
  * the library holds until the process exits.  A round that would need more
  * than ALOCO_NOALLOC_MAX_BLOCKS blocks is rejected with ALOCO_ERR_ARG and a
- * message naming both numbers; on a 152-SM GB300 the fused pass uses at most
- * 1216 blocks.  Statistics are read back with cudaMemcpyAsync into a buffer
- * on the calling thread's stack; no cudaMalloc, cudaFree, cudaMallocHost or
+ * message naming both numbers.  Every pass caps its blocks at the kernel's
+ * occupancy whatever opts->blocks_per_sm asks for: at most SMs x 8 blocks
+ * (1216 on a 152-SM GB300), so only a device with more than 256 SMs can be
+ * refused.  Statistics are read back with cudaMemcpyAsync into a buffer on
+ * the calling thread's stack; no cudaMalloc, cudaFree, cudaMallocHost or
  * other allocating routine is called.
  *
  * The first call on a device resolves the scratch array's device address
- * (cudaGetSymbolAddress, with that device current); make that first call
- * before any stream capture.  All calls on a device share the one array and
- * it keeps the previous call's contents: each call clears the counter that
- * must start at zero, and every other scratch value a round reads is
- * written by that round first.  Rounds that overlapped on the GPU would race
- * on the array; within a process the library prevents that by holding a
- * per-device lock for the whole call, which returns only after its round has
- * completed. */
+ * (cudaGetSymbolAddress, with that device current).  All calls on a device
+ * share the one array and it keeps the previous call's contents: each call
+ * clears the counter and the error word that must start at zero, and every
+ * other scratch value a round reads is written by that round first.  Rounds
+ * that overlapped on the GPU would race on the array; within a process the
+ * library prevents that by holding a per-device lock for the whole call,
+ * which returns only after its round has completed. */
 int aloco_sync_noalloc(float *global, float *momentum, void *const *locals,
                        size_t N, int M, aloco_dtype dtype, int64_t H_sel,
                        int64_t H_base, int64_t step,

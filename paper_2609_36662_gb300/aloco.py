@@ -19,6 +19,7 @@ CORR_FULL, CORR_MOMENTUM_ONLY, CORR_NONE = 0, 1, 2
 PASS_AUTO, PASS_REGISTERS, PASS_BULK_COPY = 0, 1, 2
 PASS_INT8_SPLIT, PASS_INT8_FUSED = 3, 4
 PASS_TILE = 5
+WAIT_SPIN, WAIT_BLOCK = 0, 1
 
 OK = 0
 ERR_ARG = -1
@@ -33,6 +34,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
 # Names declared in include/aloco.h (checked by the ABI test).
 EXPORTS = ("aloco_default_opts", "aloco_inner_lr_accum", "aloco_correction",
            "aloco_sync", "aloco_sync_ex", "aloco_sync_noalloc", "aloco_sync_host",
+           "aloco_sync_shard", "aloco_sync_int8_shard", "aloco_combine_partials",
            "aloco_sync_int8", "aloco_int8_num_blocks", "aloco_int8_encode",
            "aloco_int8_decode", "aloco_adamw_default_cfg", "aloco_adamw_step",
            "aloco_adamw_step_normed",
@@ -67,7 +69,7 @@ class Opts(ctypes.Structure):
                 ("time_kernel", ctypes.c_int32),
                 ("blocks_per_sm", ctypes.c_int32),
                 ("stream", ctypes.c_void_p), ("pass_", ctypes.c_int32),
-                ("reserved", ctypes.c_int32)]
+                ("wait", ctypes.c_int32)]
 
 
 class AdamwCfg(ctypes.Structure):
@@ -112,6 +114,26 @@ class Stats(ctypes.Structure):
                 "corr": self.corr.as_dict(), "nonfinite": self.nonfinite,
                 "M": self.M, "grid": self.grid, "kernel_ms": self.kernel_ms,
                 "pass_used": self.pass_used}
+
+
+class Partials(ctypes.Structure):
+    """aloco_partials_t: one shard's partial sums of a round."""
+    _fields_ = [("drift", ctypes.c_double * MAX_WORKERS),
+                ("sum_sq", ctypes.c_double), ("sq_scale", ctypes.c_double),
+                ("eps", ctypes.c_double), ("corr", Correction),
+                ("nonfinite", ctypes.c_int64), ("n", ctypes.c_int64),
+                ("M", ctypes.c_int32), ("pass_used", ctypes.c_int32),
+                ("kernel_ms", ctypes.c_float), ("reserved", ctypes.c_int32)]
+
+    def to_bytes(self) -> bytes:
+        return ctypes.string_at(ctypes.addressof(self), ctypes.sizeof(self))
+
+    @classmethod
+    def from_bytes(cls, blob: bytes) -> "Partials":
+        if len(blob) != ctypes.sizeof(cls):
+            raise ValueError(f"partials blob of {len(blob)} bytes, want "
+                             f"{ctypes.sizeof(cls)}")
+        return cls.from_buffer_copy(blob)
 
 
 _i64, _i32, _dbl = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
@@ -217,6 +239,12 @@ def load():
     lib.aloco_adamw_step_normed.restype = i32
     lib.aloco_sync_host.argtypes = sync_args + [ctypes.c_size_t, P(Opts), P(Stats)]
     lib.aloco_sync_host.restype = i32
+    lib.aloco_sync_shard.argtypes = sync_args + [P(Opts), P(Partials)]
+    lib.aloco_sync_shard.restype = i32
+    lib.aloco_sync_int8_shard.argtypes = sync_args + [vp, i32, P(Opts), P(Partials)]
+    lib.aloco_sync_int8_shard.restype = i32
+    lib.aloco_combine_partials.argtypes = [vp, i32, P(Stats)]
+    lib.aloco_combine_partials.restype = i32
     lib.aloco_test_stall_tile.argtypes = [i64]
     lib.aloco_test_stall_tile.restype = None
     lib.aloco_int8_num_blocks.argtypes = [vp, i32]
@@ -348,6 +376,71 @@ def sync(global_, momentum, locals_, *, H_sel: int, H_base: int, step: int,
 def shutdown():
     if _lib is not None:
         _lib.aloco_shutdown()
+
+
+# ------------------------------------------------------------ sharded rounds
+
+def _replica_dtype_code(t) -> int:
+    import torch
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"unsupported replica dtype {t.dtype}")
+
+
+def sync_shard(global_, momentum, locals_, *, H_sel: int, H_base: int,
+               step: int, schedule: Schedule, outer_lr: float,
+               outer_beta: float, opts: Optional[Opts] = None, stream=None,
+               raise_on_error=True, parts=None, int8: bool = False):
+    """One shard of a round on torch CUDA tensors (views of the shard's
+    elements), in place: aloco_sync_shard, or aloco_sync_int8_shard with
+    int8=True (parts: the shard's tensor parts).  Returns (status,
+    Partials)."""
+    import torch
+    N = global_.numel()
+    if momentum.numel() != N or any(x.numel() != N for x in locals_):
+        raise ValueError("all buffers must have the same number of elements")
+    for t in (global_, momentum, *locals_):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("buffers must be contiguous CUDA tensors")
+    dtype = _replica_dtype_code(locals_[0])
+    if opts is None:
+        opts = default_opts()
+    s = stream if stream is not None else torch.cuda.current_stream(
+        global_.device)
+    opts.stream = s.cuda_stream
+    M = len(locals_)
+    ptrs = (ctypes.c_void_p * M)(*[x.data_ptr() for x in locals_])
+    out = Partials()
+    with torch.cuda.device(global_.device):
+        if int8:
+            arr, n = _parts_array(parts)
+            rc = load().aloco_sync_int8_shard(
+                global_.data_ptr(), momentum.data_ptr(), ptrs, N, M, dtype,
+                H_sel, H_base, step, ctypes.byref(schedule), outer_lr,
+                outer_beta, arr, n, ctypes.byref(opts), ctypes.byref(out))
+        else:
+            rc = load().aloco_sync_shard(
+                global_.data_ptr(), momentum.data_ptr(), ptrs, N, M, dtype,
+                H_sel, H_base, step, ctypes.byref(schedule), outer_lr,
+                outer_beta, ctypes.byref(opts), ctypes.byref(out))
+    if raise_on_error and rc not in (OK, ERR_NONFINITE):
+        raise AlocoError(rc, last_error())
+    return rc, out
+
+
+def combine_partials(shards: Sequence[Partials], raise_on_error=True):
+    """aloco_combine_partials over the shards in the given order (host
+    only).  Returns the statistics dict with "status"."""
+    n = len(shards)
+    arr = (Partials * max(n, 1))(*shards)
+    st = Stats()
+    rc = load().aloco_combine_partials(arr if n else None, n,
+                                       ctypes.byref(st))
+    if raise_on_error and rc not in (OK, ERR_NONFINITE):
+        raise AlocoError(rc, last_error())
+    return st.as_dict() | {"status": rc}
 
 
 class Controller:

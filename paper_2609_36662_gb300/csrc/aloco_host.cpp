@@ -187,6 +187,7 @@ struct Workspace {
     double *stats_dev = nullptr;
     unsigned long long seq = 0;           // rounds launched on this workspace
     cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+    cudaEvent_t ev_block = nullptr;       // blocking-sync event (ALOCO_WAIT_BLOCK)
     // host-memory round (aloco_sync_host): staging slots and per-chunk totals
     char *hs = nullptr;                   // device, grown on demand
     size_t hs_cap = 0;
@@ -256,6 +257,9 @@ int ensure_ready(Workspace *ws, int device) {
     }
     if (e == cudaSuccess) e = cudaEventCreate(&ws->ev0);
     if (e == cudaSuccess) e = cudaEventCreate(&ws->ev1);
+    if (e == cudaSuccess)
+        e = cudaEventCreateWithFlags(&ws->ev_block,
+                                     cudaEventBlockingSync | cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         cudaGetLastError();
@@ -286,6 +290,21 @@ int wait_published(const double *page, unsigned long long seq, cudaStream_t stre
         }
     }
     std::atomic_thread_fence(std::memory_order_acquire);
+    return ALOCO_OK;
+}
+
+// ALOCO_WAIT_BLOCK: sleep on a blocking-sync event recorded behind the
+// kernel, then check that the round published its statistics.
+int wait_blocking(const double *page, unsigned long long seq, cudaStream_t stream,
+                  cudaEvent_t ev) {
+    cudaError_t e = cudaEventRecord(ev, stream);
+    if (e == cudaSuccess) e = cudaEventSynchronize(ev);
+    if (e != cudaSuccess) return cuda_fail(e, "round");
+    std::atomic_thread_fence(std::memory_order_acquire);
+    const volatile unsigned long long *flag =
+        reinterpret_cast<const volatile unsigned long long *>(page + aloco::kSeqSlot);
+    if (*flag != seq)
+        return fail(ALOCO_ERR_CUDA, "the round ended without publishing its statistics");
     return ALOCO_OK;
 }
 
@@ -398,6 +417,7 @@ void fill_default_opts(aloco_opts_t *o) {
     o->blocks_per_sm = 0;
     o->stream = nullptr;
     o->pass = ALOCO_PASS_AUTO;
+    o->wait = ALOCO_WAIT_SPIN;
 }
 
 // x ~= hi + lo with hi = fl32(x), lo = fl32(x - hi).
@@ -492,17 +512,37 @@ int build_parts(const int64_t *parts, int n_parts, size_t N, aloco::Int8Parts *P
     return ALOCO_OK;
 }
 
+// The partials of a shard from the round's totals block.
+void fill_partials(const double *totals, unsigned long long nf, int M, double eps,
+                   double sq_scale, const aloco_correction_t &corr, int64_t n,
+                   aloco_partials_t *p) {
+    std::memset(p, 0, sizeof *p);
+    for (int m = 0; m < M; ++m) p->drift[m] = totals ? totals[m] : 0.0;
+    p->sum_sq = totals ? totals[M] : 0.0;
+    p->sq_scale = sq_scale;
+    p->eps = eps;
+    p->corr = corr;
+    p->nonfinite = (int64_t)nf;
+    p->n = n;
+    p->M = M;
+    p->kernel_ms = -1.f;
+}
+
 // One round: the plain pass (parts == NULL && !int8) or the INT8-
-// communicated pass.
+// communicated pass.  With partials_out, the round's totals are returned
+// as a shard's partial sums instead of being finished into D and C.
 int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
               int M, aloco_dtype dtype, int64_t H_sel, int64_t H_base,
               int64_t step, const aloco_schedule_t *schedule, double outer_lr,
               double outer_beta, bool int8, const int64_t *parts, int n_parts,
-              const aloco_opts_t *opts, aloco_stats_t *stats_out) {
+              const aloco_opts_t *opts, aloco_stats_t *stats_out,
+              aloco_partials_t *partials_out = nullptr) {
     aloco_opts_t o;
     if (opts) o = *opts; else fill_default_opts(&o);
     aloco_stats_t local_stats;
     aloco_stats_t *st = stats_out ? stats_out : &local_stats;
+    if (o.wait != ALOCO_WAIT_SPIN && o.wait != ALOCO_WAIT_BLOCK)
+        return fail(ALOCO_ERR_ARG, "unknown wait mode %d", o.wait);
 
     // ---------------------------------------------------- arguments
     if (M < 1 || M > (int8 ? 16 : ALOCO_MAX_WORKERS))
@@ -534,7 +574,9 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     st->corr = corr;
     st->M = M;
     st->kernel_ms = -1.f;
+    const double sq_scale = int8 ? 1.0 : 1.0 / ((double)M * (double)M);
     if (N == 0) {
+        if (partials_out) fill_partials(nullptr, 0, M, o.eps, sq_scale, corr, 0, partials_out);
         t_err.clear();
         return ALOCO_OK;
     }
@@ -671,7 +713,10 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     if (e != cudaSuccess) return cuda_fail(e, "fused sync launch");
     if (o.time_kernel && (e = cudaEventRecord(ws->ev1, stream)) != cudaSuccess)
         return cuda_fail(e, "cudaEventRecord");
-    if ((rc = wait_published(ws->stats_host, a.seq, stream)) != ALOCO_OK) return rc;
+    rc = o.wait == ALOCO_WAIT_BLOCK
+             ? wait_blocking(ws->stats_host, a.seq, stream, ws->ev_block)
+             : wait_published(ws->stats_host, a.seq, stream);
+    if (rc != ALOCO_OK) return rc;
 
     unsigned long long nf;
     std::memcpy(&nf, ws->stats_host + aloco::kNfSlot, sizeof nf);
@@ -684,8 +729,7 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
         return fail(ALOCO_ERR_CUDA,
                     "bulk-copy pipeline wait timed out; outputs are incomplete");
     }
-    finalize_stats(ws->stats_host, nf, M, o.eps, int8 ? 1.0 : 1.0 / ((double)M * (double)M),
-                   st);
+    finalize_stats(ws->stats_host, nf, M, o.eps, sq_scale, st);
     st->grid = plan.grid;
     st->pass_used = fused ? ALOCO_PASS_INT8_FUSED
                     : int8 ? ALOCO_PASS_INT8_SPLIT
@@ -699,6 +743,16 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
             st->kernel_ms = ms;
         else
             cudaGetLastError();
+    }
+    if (partials_out) {
+        fill_partials(ws->stats_host, nf, M, o.eps, sq_scale, corr, (int64_t)N,
+                      partials_out);
+        partials_out->pass_used = st->pass_used;
+        partials_out->kernel_ms = st->kernel_ms;
+        if (nf > 0)
+            return fail(ALOCO_ERR_NONFINITE, "shard produced %llu non-finite elements", nf);
+        t_err.clear();
+        return ALOCO_OK;
     }
     if (st->nonfinite > 0 || !std::isfinite(st->D) || !std::isfinite(st->C))
         return fail(ALOCO_ERR_NONFINITE,
@@ -732,6 +786,77 @@ int aloco_sync_int8(float *global, float *momentum, void *const *locals,
     return sync_impl(global, momentum, locals, N, M, dtype, H_sel, H_base, step,
                      schedule, outer_lr, outer_beta, true, part_sizes, n_parts,
                      opts, stats_out);
+}
+
+int aloco_sync_shard(float *global, float *momentum, void *const *locals,
+                     size_t n_shard, int M, aloco_dtype dtype, int64_t H_sel,
+                     int64_t H_base, int64_t step, const aloco_schedule_t *schedule,
+                     double outer_lr, double outer_beta, const aloco_opts_t *opts,
+                     aloco_partials_t *partials_out) {
+    if (!partials_out) return fail(ALOCO_ERR_ARG, "partials_out is NULL");
+    aloco_stats_t st;
+    return sync_impl(global, momentum, locals, n_shard, M, dtype, H_sel, H_base, step,
+                     schedule, outer_lr, outer_beta, false, nullptr, 0, opts, &st,
+                     partials_out);
+}
+
+int aloco_sync_int8_shard(float *global, float *momentum, void *const *locals,
+                          size_t n_shard, int M, aloco_dtype dtype, int64_t H_sel,
+                          int64_t H_base, int64_t step, const aloco_schedule_t *schedule,
+                          double outer_lr, double outer_beta, const int64_t *part_sizes,
+                          int n_parts, const aloco_opts_t *opts,
+                          aloco_partials_t *partials_out) {
+    if (!partials_out) return fail(ALOCO_ERR_ARG, "partials_out is NULL");
+    aloco_stats_t st;
+    return sync_impl(global, momentum, locals, n_shard, M, dtype, H_sel, H_base, step,
+                     schedule, outer_lr, outer_beta, true, part_sizes, n_parts, opts, &st,
+                     partials_out);
+}
+
+int aloco_combine_partials(const aloco_partials_t *shards, int n_shards,
+                           aloco_stats_t *stats_out) {
+    if (!shards || n_shards < 1) return fail(ALOCO_ERR_ARG, "need n_shards >= 1 partials");
+    if (!stats_out) return fail(ALOCO_ERR_ARG, "stats_out is NULL");
+    const aloco_partials_t &p0 = shards[0];
+    const int M = p0.M;
+    if (M < 1 || M > ALOCO_MAX_WORKERS)
+        return fail(ALOCO_ERR_ARG, "shard 0: M = %d outside [1, %d]", M, ALOCO_MAX_WORKERS);
+    for (int k = 1; k < n_shards; ++k) {
+        const aloco_partials_t &p = shards[k];
+        if (p.M != M || p.eps != p0.eps || p.sq_scale != p0.sq_scale ||
+            std::memcmp(&p.corr, &p0.corr, sizeof p.corr) != 0)
+            return fail(ALOCO_ERR_ARG,
+                        "shard %d does not belong to the round of shard 0 (M, eps, "
+                        "aggregate scale or correction context differ)", k);
+    }
+    // fixed shard order: every holder adds the same values in the same order
+    double tot[ALOCO_MAX_WORKERS + 1] = {};
+    unsigned long long nf = 0;
+    float ms = -1.f;
+    int pass_used = 0;
+    for (int k = 0; k < n_shards; ++k) {
+        const aloco_partials_t &p = shards[k];
+        if (p.nonfinite < 0) return fail(ALOCO_ERR_ARG, "shard %d: negative count", k);
+        for (int m = 0; m < M; ++m) tot[m] += p.drift[m];
+        tot[M] += p.sum_sq;
+        nf += (unsigned long long)p.nonfinite;
+        if (p.kernel_ms > ms) ms = p.kernel_ms;
+        if (!pass_used && p.n > 0) pass_used = p.pass_used;
+    }
+    std::memset(stats_out, 0, sizeof *stats_out);
+    finalize_stats(tot, nf, M, p0.eps, p0.sq_scale, stats_out);
+    stats_out->corr = p0.corr;
+    stats_out->M = M;
+    stats_out->grid = n_shards;
+    stats_out->kernel_ms = ms;
+    stats_out->pass_used = pass_used;
+    if (stats_out->nonfinite > 0 || !std::isfinite(stats_out->D) ||
+        !std::isfinite(stats_out->C))
+        return fail(ALOCO_ERR_NONFINITE,
+                    "combined round has %lld non-finite elements (D=%g, C=%g)",
+                    (long long)stats_out->nonfinite, stats_out->D, stats_out->C);
+    t_err.clear();
+    return ALOCO_OK;
 }
 
 int64_t aloco_int8_num_blocks(const int64_t *part_sizes, int n_parts) {
@@ -1316,6 +1441,8 @@ void aloco_shutdown(void) {
         cudaDeviceSynchronize();
         if (ws->ev0) cudaEventDestroy(ws->ev0);
         if (ws->ev1) cudaEventDestroy(ws->ev1);
+        if (ws->ev_block) cudaEventDestroy(ws->ev_block);
+        ws->ev_block = nullptr;
         if (ws->host) cudaFreeHost(ws->host);
         if (ws->stats_host) cudaFreeHost(ws->stats_host);
         if (ws->dev) cudaFree(ws->dev);

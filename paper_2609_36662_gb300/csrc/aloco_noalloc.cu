@@ -7,12 +7,15 @@
 // and hand it out from their own pools, deployments whose memory footprint
 // must be fixed when the library is loaded, and loops that cannot afford the
 // implicit device synchronisation of cudaMalloc / cudaFree.  For them this
-// entry point runs the same fused kernel with its scratch (per-block partial
-// sums, the last-block ticket and the totals) in a file-scope __device__
-// array that exists, on every device that loads the library, from module load
-// until the process exits.  It calls no cudaMalloc, cudaFree, cudaMallocHost
-// or other allocating routine; the statistics come back through a plain
-// cudaMemcpyAsync into a buffer on the caller's stack.
+// entry point runs the same fused kernel as aloco_sync_ex, chosen by the same
+// rule (the tile pass, the bulk-copy pass or the register pass) and launched
+// with the same grid, with its scratch (per-block partial sums, the
+// last-block ticket and the totals) in a file-scope __device__ array that
+// exists, on every device that loads the library, from module load until the
+// process exits.  It calls no cudaMalloc, cudaFree, cudaMallocHost or other
+// allocating routine; the statistics come back through a plain
+// cudaMemcpyAsync into a buffer on the caller's stack, followed by a stream
+// synchronisation, so a call cannot be part of a stream capture.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -27,8 +30,11 @@
 namespace {
 
 // Block partials the scratch can hold: one row of M + 1 fp64 values per
-// block.  The fused pass never uses more blocks than SMs x 8 (256-thread
-// blocks, 2048 threads per SM), i.e. 1216 on a 152-SM GB300.
+// block.  The register and bulk-copy passes cap their residency at the
+// kernel's occupancy, whatever opts->blocks_per_sm asks for, so they use at
+// most SMs x 8 blocks (256-thread blocks, 2048 threads per SM); the tile
+// pass uses at most SMs x 4.  On a 152-SM GB300 that is 1216 rows; only a
+// device with more than 256 SMs could be refused.
 constexpr int kScratchBlocks = ALOCO_NOALLOC_MAX_BLOCKS;
 
 struct NoallocScratch {
@@ -146,6 +152,21 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
         cudaGetLastError();
         return errf(ALOCO_ERR_CUDA, "cudaGetDevice failed or device out of range");
     }
+    cudaStream_t stream = (cudaStream_t)o.stream;
+    {
+        // the call ends with a stream synchronisation, which a capture
+        // cannot contain: refuse before any other CUDA call
+        cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+        e = cudaStreamIsCapturing(stream, &cap);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return errf(ALOCO_ERR_CUDA, "cudaStreamIsCapturing: %s", cudaGetErrorString(e));
+        }
+        if (cap != cudaStreamCaptureStatusNone)
+            return errf(ALOCO_ERR_ARG,
+                        "aloco_sync_noalloc cannot run under stream capture: it "
+                        "waits for its round with a stream synchronisation");
+    }
     std::lock_guard<std::mutex> lk(g_mu[device]);
     if ((rc = setup_device(device)) != ALOCO_OK) return rc;
     if ((rc = aloco::check_buffer(global, N * 4, device, "global")) != ALOCO_OK)
@@ -178,8 +199,16 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
 
     const int64_t work = a.nvec > 0 ? a.nvec : a.n;
     aloco::LaunchPlan plan;
-    const bool tma = aloco::use_tma(o.pass, M, dtype, a.nvec);
-    if (tma)
+    // the same choice of kernel as aloco_sync_ex
+    const bool tile = aloco::use_tile(o.pass, M, dtype, a.n, a.nvec);
+    const bool tma = !tile && aloco::use_tma(o.pass, M, dtype, a.nvec);
+    plan.grid = 0;
+    plan.block = 0;
+    plan.kernel = nullptr;
+    e = cudaSuccess;
+    if (tile)
+        ;  // launch_sync_tile picks its grid below (at most SMs x 4 CTAs)
+    else if (tma)
         e = dtype == ALOCO_F32
                 ? aloco::plan_sync_tma_f32(M, a.nvec, g_sms[device], &plan)
                 : aloco::plan_sync_tma_bf16(M, a.nvec, g_sms[device], &plan);
@@ -207,7 +236,6 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
     a.n_tiles = plan.tiles;
     a.stages = plan.stages;
 
-    cudaStream_t stream = (cudaStream_t)o.stream;
     // The ticket and the error word must start at zero; every partial row
     // and total used by this launch is written by it before it is read.
     e = cudaMemsetAsync(&s->ticket, 0, sizeof(unsigned int), stream);
@@ -217,9 +245,14 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
         cudaGetLastError();
         return errf(ALOCO_ERR_CUDA, "ticket reset: %s", cudaGetErrorString(e));
     }
-    void *params[] = {&a};
-    e = cudaLaunchKernel(plan.kernel, dim3(plan.grid), dim3(plan.block), params,
-                         plan.smem, stream);
+    if (tile) {
+        e = aloco::launch_sync_tile(a, dtype, g_sms[device], kScratchBlocks, stream,
+                                    &plan.grid);
+    } else {
+        void *params[] = {&a};
+        e = cudaLaunchKernel(plan.kernel, dim3(plan.grid), dim3(plan.block), params,
+                             plan.smem, stream);
+    }
     if (e != cudaSuccess) {
         cudaGetLastError();
         return errf(ALOCO_ERR_CUDA, "fused sync launch: %s", cudaGetErrorString(e));
@@ -241,7 +274,7 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
                     "bulk-copy pipeline wait timed out; outputs are incomplete");
     aloco::finalize_stats(host, nf, M, o.eps, 1.0 / ((double)M * (double)M), st);
     st->grid = plan.grid;
-    st->pass_used = tma ? ALOCO_PASS_BULK_COPY : ALOCO_PASS_REGISTERS;
+    st->pass_used = tile ? ALOCO_PASS_TILE : tma ? ALOCO_PASS_BULK_COPY : ALOCO_PASS_REGISTERS;
     if (st->nonfinite > 0 || !std::isfinite(st->D) || !std::isfinite(st->C))
         return errf(ALOCO_ERR_NONFINITE,
                     "round produced %lld non-finite elements (D=%g, C=%g)",

@@ -205,23 +205,51 @@ def n_chunks(w: Workload) -> int:
     return (w.numel + CHUNK - 1) // CHUNK
 
 
-def make_global(w: Workload, device="cpu", draw: int = 0):
+def make_global(w: Workload, device="cpu", draw: int = 0,
+                upto: Optional[int] = None, chunks: Optional[Tuple[int, int]] = None):
     """theta_global ~ N(0, 0.02) (fp32); norm vectors set to 1.0.  `draw`
-    selects an independent draw of the same distribution."""
-    g = torch.empty(w.numel, dtype=torch.float32, device=device)
+    selects an independent draw of the same distribution.  With `upto`,
+    only the whole generator chunks that cover elements [0, upto) are drawn
+    (a prefix of the same vector); with `chunks` = (c_lo, c_hi), only the
+    elements of generator chunks c_lo .. c_hi - 1 (a contiguous piece of the
+    same vector, starting at element c_lo * CHUNK)."""
+    if chunks is None:
+        c_lo = 0
+        c_hi = n_chunks(w) if upto is None else min(n_chunks(w), n_chunks_upto(upto))
+    else:
+        c_lo, c_hi = chunks
+    base = c_lo * CHUNK
+    end = min(w.numel, c_hi * CHUNK)
+    g = torch.empty(max(end - base, 0), dtype=torch.float32, device=device)
     key = 0 if draw == 0 else 10_000 + draw
-    for c in range(n_chunks(w)):
+    for c in range(c_lo, c_hi):
         s, e = c * CHUNK, min(w.numel, (c + 1) * CHUNK)
-        g[s:e].normal_(0.0, 0.02, generator=_chunk_gen(device, w.seed, key, c))
+        g[s - base:e - base].normal_(0.0, 0.02,
+                                     generator=_chunk_gen(device, w.seed, key, c))
     if w.shape is not None:
-        for off, n, _, is_norm in _segments(w):
-            if is_norm:
-                g[off:off + n] = 1.0
+        for off, k, _, is_norm in _segments(w):
+            lo, hi = max(off, base), min(off + k, end)
+            if is_norm and lo < hi:
+                g[lo - base:hi - base] = 1.0
     return g
 
 
-def make_momentum(w: Workload, device="cpu"):
-    return torch.zeros(w.numel, dtype=torch.float32, device=device)
+def n_chunks_upto(upto: int) -> int:
+    """Generator chunks that cover elements [0, upto)."""
+    return (max(upto, 1) + CHUNK - 1) // CHUNK
+
+
+def make_momentum(w: Workload, device="cpu", upto: Optional[int] = None):
+    n = w.numel if upto is None else min(w.numel, n_chunks_upto(upto) * CHUNK)
+    return torch.zeros(n, dtype=torch.float32, device=device)
+
+
+def shard_chunks(w: Workload, shards: int, k: int) -> Tuple[int, int]:
+    """Generator chunks [c_lo, c_hi) of shard k when the vector is cut into
+    `shards` contiguous pieces at chunk boundaries (near-equal chunk counts;
+    a shard may be empty when there are more shards than chunks)."""
+    nc = n_chunks(w)
+    return nc * k // shards, nc * (k + 1) // shards
 
 
 def replica_dtype(w: Workload):

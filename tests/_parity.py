@@ -366,3 +366,95 @@ def oracle_stats_host_threaded(w: W.Workload, g_h, x_h, eps=1e-8,
         B += acc.B.value
     D = sum(E) / w.M
     return {"D": D, "C": w.M * B / (D + eps), "mean_sq_norm": B, "drift": E}
+
+
+
+class _FieldCheck:
+    """Streaming form of the field tolerance over a vector seen slice by
+    slice: the bound excess <= rtol * max(|field|, rms(field)) needs the
+    whole field's rms, so elements whose excess is above rtol * |field| are
+    kept as candidates and judged against the rms once every slice has been
+    seen."""
+
+    def __init__(self, name, rtol=RTOL_FIELD):
+        self.name, self.rtol = name, rtol
+        self.sq, self.n = 0.0, 0
+        self.excess, self.ref, self.index = [], [], []
+
+    def add(self, excess, field, offset):
+        field = np.asarray(field, np.float64)
+        self.sq += float(np.dot(field, field))
+        self.n += field.size
+        a = np.abs(field)
+        c = np.nonzero(excess > self.rtol * a)[0]
+        self.excess.append(excess[c])
+        self.ref.append(a[c])
+        self.index.append(c + offset)
+
+    def check(self) -> int:
+        """Assert the bound; returns the number of elements that needed the
+        rms part of it."""
+        rms = np.sqrt(self.sq / max(self.n, 1))
+        ex = np.concatenate(self.excess)
+        ref = np.concatenate(self.ref)
+        idx = np.concatenate(self.index)
+        bad = ex > self.rtol * np.maximum(ref, rms)
+        assert not bad.any(), (f"{self.name}: {int(bad.sum())} elements beyond "
+                               f"the field tolerance, e.g. index "
+                               f"{int(idx[np.argmax(bad)])}")
+        return int(ex.size)
+
+
+def _abs_diff(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    d = np.abs(a - b)
+    d[a == b] = 0.0
+    return d
+
+
+def compare_whole_vector(w: W.Workload, g_in, v_in, x_in, g, v, xs, corr,
+                         slice_elems=1 << 24, threads=16):
+    """theta', v' and the replica reset of a round against the oracle's
+    elementwise update over the WHOLE vector (not a sample), slice by slice:
+    each slice of the device snapshot of the inputs and of the GPU's outputs
+    is copied to the host, the oracle's pass 2 runs on it in threads, and
+    every element is held to the tolerances of compare_round.  Host memory
+    stays at a few slices whatever the vector's size.  The replica reset is
+    compared with the oracle through replica 0; the caller checks on the
+    device that every replica equals it (the reset writes one value)."""
+    N = w.numel
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+    fg, fv, fx = (_FieldCheck("theta'"), _FieldCheck("v'"),
+                  _FieldCheck("replica 0"))
+    sub = max(1, slice_elems // threads)
+    for s in range(0, N, slice_elems):
+        e = min(N, s + slice_elems)
+        gh = g_in[s:e].cpu().numpy()
+        vh = v_in[s:e].cpu().numpy()
+        xh = [to_numpy_bits(x[s:e]) for x in x_in]
+        go = np.empty(e - s, np.float64)
+        vo = np.empty(e - s, np.float64)
+        xo = np.empty(e - s, np.float32 if dt == O.F32 else np.uint16)
+
+        def work(a):
+            b = min(e - s, a + sub)
+            r = O.pass2(gh[a:b], vh[a:b], [x[a:b] for x in xh], dt,
+                        corr.mu_t, corr.eta_out, corr.inv_norm,
+                        want_replicas=True)
+            go[a:b], vo[a:b], xo[a:b] = r[0], r[1], r[2][0]
+
+        with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+            list(ex.map(work, range(0, e - s, sub)))
+        fg.add(_abs_diff(g[s:e].cpu().numpy(), go), go, s)
+        fv.add(_abs_diff(v[s:e].cpu().numpy(), vo), vo, s)
+        x0 = to_numpy_bits(xs[0][s:e])
+        if dt == O.F32:
+            fx.add(_abs_diff(x0, xo), xo, s)
+        else:
+            # one bf16 ulp at the oracle's value, then theta's own bound
+            ov = O.bf16_bits_to_float(xo)
+            fx.add(_abs_diff(O.bf16_bits_to_float(x0), ov) - bf16_ulp(ov),
+                   go, s)
+    return {"theta_candidates": fg.check(), "v_candidates": fv.check(),
+            "replica_candidates": fx.check()}
