@@ -31,11 +31,12 @@
 // arithmetic of every element is the split form's (aloco_int8.cu), so both
 // forms give the same codes, scales and outputs.
 //
-// Shared memory per CTA: the input buffer, 4096 x (8 + M x element size)
-// bytes, and the output tiles, 4096 x element size (plus 4096 x 8 for the
-// fp32 theta' and v' tiles where they fit; elsewhere threads store theta'
-// and v' themselves).  It holds M <= 8 fp32 or M <= 16 bf16 replicas;
-// larger worker counts use the split form.
+// Shared memory per CTA: the input buffer, 4096 x (8 + G x element size)
+// bytes for a group of G workers, and the output tiles, 4096 x element size
+// (plus 4096 x 8 for the fp32 theta' and v' tiles where they fit; elsewhere
+// threads store theta' and v' themselves).  One group holds every worker for
+// bf16 and for fp32 up to M = 8; fp32 with 9 <= M <= 16 stages each block's
+// replicas in groups of about three workers (see fused_group).
 //
 // A bounded wait that runs out (about 2 s) sets the round's error word; the
 // whole CTA leaves the block loop together at the next barrier, thread 0

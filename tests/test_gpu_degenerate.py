@@ -8,7 +8,11 @@
     all zero (scale 1, codes 0), so the decoded aggregate is 0 as well.
   * Identical replicas: every worker returns the same endpoint x != theta.
     Then every ||Delta_m||^2 is the same value, ||Dbar||^2 = D and
-    C = M D / (D + eps), just below M, the top of the range 0 <= C < M.
+    C = M D / (D + eps), just below M, the top of the range 0 <= C < M
+    (up to the fp32 rounding of the sum over workers).  In the INT8 round
+    C comes from the decoded aggregate and D from the raw pseudo-gradients
+    (App. G.1), so there C differs from M D / (D + eps) by the codec's
+    error and only the oracle comparison and the equal energies apply.
 
 Each case runs on the register, bulk-copy and tile passes of the plain
 round and on both forms of the INT8 round, for both replica types, on a
@@ -29,7 +33,8 @@ pytestmark = pytest.mark.gpu
 N = 1_000_003
 PLAIN = {"registers": A.PASS_REGISTERS, "bulk_copy": A.PASS_BULK_COPY,
          "tile": A.PASS_TILE}
-INT8 = {"int8_split": A.PASS_INT8_SPLIT, "int8_fused": A.PASS_INT8_FUSED}
+INT8 = {"int8_split": A.PASS_INT8_SPLIT, "int8_fused": A.PASS_INT8_FUSED,
+        "int8_pipelined": A.PASS_INT8_PIPELINED}
 INT8_PARTS = [3 * 4096 + 64, 768, 5001, 12, 4096, N - (3 * 4096 + 64 + 768 +
                                                        5001 + 12 + 4096)]
 
@@ -68,7 +73,7 @@ def _round(w, g, v, xs, pass_):
     return A.sync(g, v, xs, **kw)
 
 
-def _check_case(w, case, st, g_in, v_in, g, v):
+def _check_case(w, case, st, g_in, v_in, g, v, int8=False):
     M = w.M
     if case == "zero_drift":
         assert st["D"] == 0.0 and st["C"] == 0.0
@@ -83,9 +88,10 @@ def _check_case(w, case, st, g_in, v_in, g, v):
         d = st["drift"]
         assert all(x == d[0] for x in d), "identical workers, unequal energies"
         assert d[0] > 0.0
-        assert_rel(st["C"], M * st["D"] / (st["D"] + 1e-8), "C vs M D/(D+eps)",
-                   RTOL_STAT)
-        assert st["C"] < M
+        if not int8:
+            assert_rel(st["C"], M * st["D"] / (st["D"] + 1e-8),
+                       "C vs M D/(D+eps)", RTOL_STAT)
+            assert st["C"] < M * (1 + RTOL_STAT)
 
 
 @pytest.mark.parametrize("case", ["zero_drift", "identical"])
@@ -109,6 +115,8 @@ def test_plain_round_degenerate_cases(case, pass_name, dt, M):
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
 @pytest.mark.parametrize("M", [1, 4, 8, 16])
 def test_int8_round_degenerate_cases(case, form, dt, M):
+    if form == "int8_pipelined" and (dt != "bf16" or M < 2):
+        pytest.skip("the pipelined form takes bf16 replicas and M >= 2")
     w = W.small(N, M, dt, seed=95 + M)
     g, v, xs = _state(w, case)
     g_in, v_in = g.clone(), v.clone()
@@ -122,4 +130,4 @@ def test_int8_round_degenerate_cases(case, form, dt, M):
     assert st["status"] == A.OK, A.last_error()
     assert st["pass_used"] == INT8[form]
     compare_round(w, st, orc, g, v, xs)
-    _check_case(w, case, st, g_in, v_in, g, v)
+    _check_case(w, case, st, g_in, v_in, g, v, int8=True)

@@ -97,7 +97,13 @@ def _fits_fused(dt, M):
     return M <= 16
 
 
-FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
+FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED,
+         "pipelined": A.PASS_INT8_PIPELINED}
+
+
+def _form_applies(form, dt, M):
+    """The pipelined form takes bf16 replicas and 2 <= M <= 16."""
+    return form != "pipelined" or (dt == "bf16" and 2 <= M <= 16)
 
 
 @pytest.mark.parametrize("form", sorted(FORMS))
@@ -107,6 +113,8 @@ FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
 def test_int8_round_matches_oracle(dt, M, parts_name, form):
     if form == "fused" and not _fits_fused(dt, M):
         pytest.skip("the fused form holds M <= 16")
+    if not _form_applies(form, dt, M):
+        pytest.skip("the pipelined form takes bf16 replicas and M >= 2")
     parts = PARTS[parts_name]
     N = sum(parts) if parts else 5 * 4096 + 333
     w = W.small(N, M, dt, seed=40 + M)
@@ -126,15 +134,17 @@ def test_int8_round_matches_oracle(dt, M, parts_name, form):
                                   ("bf16", 5), ("bf16", 8), ("bf16", 9), ("bf16", 12),
                                   ("bf16", 16), ("f32", 9), ("f32", 12), ("f32", 16)])
 def test_int8_forms_agree_bit_for_bit(dt, M):
-    """The fused and the split form take the same decisions in the same
-    arithmetic: theta', v' and the replicas are bit-identical; the
-    statistics agree within the statistics tolerance (the forms group each
-    thread's fp32 partial energies differently)."""
+    """The forms take the same decisions in the same arithmetic: theta', v'
+    and the replicas are bit-identical; the statistics agree within the
+    statistics tolerance (the forms group each thread's fp32 partial
+    energies differently)."""
     parts = PARTS["llama_like"]
     w = W.small(sum(parts), M, dt, seed=70 + M)
     sa, _ = schedule_pair(w.schedule)
     out = {}
     for form, p in FORMS.items():
+        if not _form_applies(form, dt, M):
+            continue
         g, v, xs = gpu_inputs(w)
         v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(M))
         st = A.sync_int8(g, v, xs, parts=parts, H_sel=w.H_sel[0],
@@ -150,6 +160,15 @@ def test_int8_forms_agree_bit_for_bit(dt, M):
     for key in ("D", "C", "mean_sq_norm"):
         assert s1[key] == pytest.approx(s2[key], rel=RTOL_STAT), key
     assert s1["nonfinite"] == s2["nonfinite"] == 0
+    if "pipelined" in out:
+        s3, g3, v3, x3 = out["pipelined"]
+        assert s3["pass_used"] == A.PASS_INT8_PIPELINED
+        assert torch.equal(g3.view(torch.int32), g2.view(torch.int32))
+        assert torch.equal(v3.view(torch.int32), v2.view(torch.int32))
+        for a, b in zip(x3, x2):
+            assert torch.equal(a, b)
+        for key in ("D", "C", "mean_sq_norm"):
+            assert s3[key] == pytest.approx(s2[key], rel=RTOL_STAT), key
 
 
 def test_int8_auto_form():
