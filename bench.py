@@ -47,7 +47,7 @@ UNIT = "rounds/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 PASSES = {"auto": 0, "registers": 1, "bulk_copy": 2, "int8_split": 3,
-          "int8_fused": 4, "tile": 5, "int8_pipelined": 6}
+          "int8_fused": 4, "tile": 5}
 
 
 def workloads_by_name():
@@ -152,8 +152,6 @@ KERNEL_SOURCES = {
                            "aloco_int8.cu"),
     "int8_fused_kernel": ("aloco_sync_kernel.cuh", "aloco_bulk.cuh", "aloco_int8.cuh",
                           "aloco_int8_fused.cu"),
-    "int8_pipelined_kernel": ("aloco_sync_kernel.cuh", "aloco_bulk.cuh", "aloco_int8.cuh",
-                              "aloco_int8_pipelined.cu"),
     "adamw_kernels": ("aloco_sync_kernel.cuh", "aloco_adamw.cu"),
 }
 
@@ -608,8 +606,7 @@ def run_cuda(args, w):
         step_ms.append(ev[k][0].elapsed_time(ev[k][1]))
 
     kernel_name = {2: "sync_tma_kernel", 3: "int8_split_kernels",
-                   4: "int8_fused_kernel", 5: "sync_tile_kernel",
-                   6: "int8_pipelined_kernel"}.get(st_first.get("pass_used"),
+                   4: "int8_fused_kernel", 5: "sync_tile_kernel"}.get(st_first.get("pass_used"),
                                                "sync_kernel")
     # median over the timed rounds (each rank), then the slowest rank
     ms_step_mean = reduce_max(statistics.mean(step_ms), world, device)

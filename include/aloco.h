@@ -128,13 +128,8 @@ typedef enum {
  *              replicas in shared memory, reading every replica once
  *              (any M <= 16; above 8 fp32 replicas it stages each
  *              block's replicas in groups);
- *   INT8_PIPELINED  bf16 replicas, 2 <= M <= 16: the fused form with one
- *              shared-memory slot per worker that is refilled with the next
- *              block as soon as every warp has read it, so the next block's
- *              copies overlap this block's codec work (other shapes:
- *              ALOCO_ERR_ARG);
  *   AUTO       the form measured faster on GB300 for (M, dtype).
- * The three INT8 forms give the same theta', v' and replicas bit for bit.
+ * The two INT8 forms give the same theta', v' and replicas bit for bit.
  * aloco_sync / aloco_sync_ex reject the INT8 values and aloco_sync_int8 the
  * REGISTERS / BULK_COPY / TILE values with ALOCO_ERR_ARG. */
 typedef enum {
@@ -143,8 +138,7 @@ typedef enum {
     ALOCO_PASS_BULK_COPY = 2,
     ALOCO_PASS_INT8_SPLIT = 3,
     ALOCO_PASS_INT8_FUSED = 4,
-    ALOCO_PASS_TILE = 5,
-    ALOCO_PASS_INT8_PIPELINED = 6
+    ALOCO_PASS_TILE = 5
 } aloco_pass;
 
 /* How a round call waits for its kernel (aloco_sync_ex, aloco_sync_int8 and

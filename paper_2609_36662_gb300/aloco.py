@@ -19,7 +19,6 @@ CORR_FULL, CORR_MOMENTUM_ONLY, CORR_NONE = 0, 1, 2
 PASS_AUTO, PASS_REGISTERS, PASS_BULK_COPY = 0, 1, 2
 PASS_INT8_SPLIT, PASS_INT8_FUSED = 3, 4
 PASS_TILE = 5
-PASS_INT8_PIPELINED = 6
 WAIT_SPIN, WAIT_BLOCK = 0, 1
 
 OK = 0

@@ -112,7 +112,7 @@ int correction_impl(const aloco_schedule_t *sched, int64_t step,
     if (!std::isfinite(outer_lr)) return fail(ALOCO_ERR_ARG, "outer_lr must be finite");
     if (o.blocks_per_sm < 0)
         return fail(ALOCO_ERR_ARG, "blocks_per_sm must be >= 0");
-    if (o.pass < ALOCO_PASS_AUTO || o.pass > ALOCO_PASS_INT8_PIPELINED)
+    if (o.pass < ALOCO_PASS_AUTO || o.pass > ALOCO_PASS_TILE)
         return fail(ALOCO_ERR_ARG, "unknown pass %d", o.pass);
     if (o.mode != ALOCO_CORR_FULL && o.mode != ALOCO_CORR_MOMENTUM_ONLY &&
         o.mode != ALOCO_CORR_NONE)
@@ -339,23 +339,11 @@ namespace aloco {
 
 bool use_int8_fused(int pass, int M, aloco_dtype dtype) {
     if (!int8_fused_fits(M, dtype)) return false;
-    if (pass == ALOCO_PASS_INT8_FUSED || pass == ALOCO_PASS_INT8_PIPELINED) return true;
+    if (pass == ALOCO_PASS_INT8_FUSED) return true;
     if (pass == ALOCO_PASS_INT8_SPLIT) return false;
     return true;  // AUTO
 }
 
-// Worker counts from which AUTO takes the pipelined form for bf16 replicas
-// (a tuning knob: 17 keeps AUTO on the fused form).
-#ifndef ALOCO_I8_PIPE_MIN
-#define ALOCO_I8_PIPE_MIN 17
-#endif
-
-bool use_int8_pipelined(int pass, int M, aloco_dtype dtype) {
-    if (!int8_pipelined_fits(M, dtype)) return false;
-    if (pass == ALOCO_PASS_INT8_PIPELINED) return true;
-    if (pass != ALOCO_PASS_AUTO) return false;
-    return M >= ALOCO_I8_PIPE_MIN;
-}
 
 bool use_tile(int pass, int M, aloco_dtype dtype, int64_t n, int64_t nvec) {
     if (!sync_tile_fits(M, n, nvec)) return false;
@@ -563,17 +551,13 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
                     int8 ? 16 : ALOCO_MAX_WORKERS);
     if (dtype != ALOCO_F32 && dtype != ALOCO_BF16)
         return fail(ALOCO_ERR_ARG, "unknown replica dtype %d", (int)dtype);
-    const bool int8_pass = o.pass == ALOCO_PASS_INT8_SPLIT || o.pass == ALOCO_PASS_INT8_FUSED ||
-                           o.pass == ALOCO_PASS_INT8_PIPELINED;
+    const bool int8_pass = o.pass == ALOCO_PASS_INT8_SPLIT || o.pass == ALOCO_PASS_INT8_FUSED;
     if (int8 ? (o.pass == ALOCO_PASS_REGISTERS || o.pass == ALOCO_PASS_BULK_COPY ||
                 o.pass == ALOCO_PASS_TILE)
              : int8_pass)
         return fail(ALOCO_ERR_ARG, "pass %d does not apply to this round", o.pass);
     if (int8 && o.pass == ALOCO_PASS_INT8_FUSED && !aloco::int8_fused_fits(M, dtype))
         return fail(ALOCO_ERR_ARG, "the fused INT8 round takes M <= 16");
-    if (int8 && o.pass == ALOCO_PASS_INT8_PIPELINED && !aloco::int8_pipelined_fits(M, dtype))
-        return fail(ALOCO_ERR_ARG,
-                    "the pipelined INT8 round takes bf16 replicas and 2 <= M <= 16");
     if (N > (size_t)INT64_MAX / 8) return fail(ALOCO_ERR_ARG, "N too large");
     if (N > 0 && (!global || !momentum || !locals))
         return fail(ALOCO_ERR_ARG, "NULL buffer");
@@ -663,7 +647,6 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     const bool tile = !int8 && aloco::use_tile(o.pass, M, dtype, a.n, a.nvec);
     const bool tma = !int8 && !tile && aloco::use_tma(o.pass, M, dtype, a.nvec);
     const bool fused = int8 && aloco::use_int8_fused(o.pass, M, dtype);
-    const bool piped = fused && aloco::use_int8_pipelined(o.pass, M, dtype);
     if (fused || tile) {
         plan.grid = 0;
         plan.block = 0;
@@ -712,10 +695,7 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     cudaStream_t stream = (cudaStream_t)o.stream;
     if (o.time_kernel && (e = cudaEventRecord(ws->ev0, stream)) != cudaSuccess)
         return cuda_fail(e, "cudaEventRecord");
-    if (piped) {
-        e = aloco::launch_int8_pipelined(a, P, dtype, ws->sm_count, ws->max_grid, stream,
-                                         &plan.grid);
-    } else if (fused) {
+    if (fused) {
         e = aloco::launch_int8_fused(a, P, dtype, ws->sm_count, ws->max_grid, stream,
                                      &plan.grid);
     } else if (tile) {
@@ -752,8 +732,7 @@ int sync_impl(float *global, float *momentum, void *const *locals, size_t N,
     }
     finalize_stats(ws->stats_host, nf, M, o.eps, sq_scale, st);
     st->grid = plan.grid;
-    st->pass_used = piped ? ALOCO_PASS_INT8_PIPELINED
-                    : fused ? ALOCO_PASS_INT8_FUSED
+    st->pass_used = fused ? ALOCO_PASS_INT8_FUSED
                     : int8 ? ALOCO_PASS_INT8_SPLIT
                     : tile ? ALOCO_PASS_TILE
                     : tma  ? ALOCO_PASS_BULK_COPY

@@ -146,12 +146,6 @@ bool int8_fused_fits(int M, aloco_dtype dtype);
 cudaError_t launch_int8_fused(const SyncArgs &a, const Int8Parts &P,
                               aloco_dtype dtype, int sm_count, int max_grid,
                               cudaStream_t stream, int *grid_out);
-// The pipelined fused form (aloco_int8_pipelined.cu): bf16, 2 <= M <= 16.
-bool int8_pipelined_fits(int M, aloco_dtype dtype);
-bool use_int8_pipelined(int pass, int M, aloco_dtype dtype);
-cudaError_t launch_int8_pipelined(const SyncArgs &a, const Int8Parts &P,
-                                  aloco_dtype dtype, int sm_count, int max_grid,
-                                  cudaStream_t stream, int *grid_out);
 cudaError_t launch_int8_encode(const float *x, int8_t *codes, float *scales,
                                float *decoded, bool vec_ok, const Int8Parts &P,
                                int sm_count, cudaStream_t stream);

@@ -105,8 +105,7 @@ extern "C" int aloco_sync_noalloc(float *global, float *momentum,
         return errf(ALOCO_ERR_ARG, "M = %d outside [1, %d]", M, ALOCO_MAX_WORKERS);
     if (dtype != ALOCO_F32 && dtype != ALOCO_BF16)
         return errf(ALOCO_ERR_ARG, "unknown replica dtype %d", (int)dtype);
-    if (o.pass == ALOCO_PASS_INT8_SPLIT || o.pass == ALOCO_PASS_INT8_FUSED ||
-        o.pass == ALOCO_PASS_INT8_PIPELINED)
+    if (o.pass == ALOCO_PASS_INT8_SPLIT || o.pass == ALOCO_PASS_INT8_FUSED)
         return errf(ALOCO_ERR_ARG, "pass %d does not apply to this round", o.pass);
     if (N > (size_t)INT64_MAX / 8) return errf(ALOCO_ERR_ARG, "N too large");
     if (N > 0 && (!global || !momentum || !locals))

@@ -227,7 +227,7 @@ def test_pass_values_are_checked_against_the_round(lib):
     s = A.Schedule.make()
     base = 1 << 40
     xs = [base + (k + 2) * (1 << 22) for k in range(2)]
-    for p in (A.PASS_INT8_SPLIT, A.PASS_INT8_FUSED, A.PASS_INT8_PIPELINED, 7, -1):
+    for p in (A.PASS_INT8_SPLIT, A.PASS_INT8_FUSED, 6, -1):
         for noalloc in (False, True):
             rc, _ = A.sync_ptrs(base, base + (1 << 22), xs, 1000, A.F32, 150,
                                 100, 4000, s, 0.7, 0.9,
@@ -255,11 +255,6 @@ def test_pass_values_are_checked_against_the_round(lib):
     # accepted combinations get past argument checks (no device here)
     assert int8(4, A.F32, A.PASS_INT8_FUSED) in (A.ERR_CUDA, A.ERR_ARG)
     assert "fused" not in A.last_error()
-    # the pipelined form takes bf16 replicas and 2 <= M <= 16
-    for M, dt in ((4, A.F32), (1, A.BF16), (17, A.BF16)):
-        assert int8(M, dt, A.PASS_INT8_PIPELINED) == A.ERR_ARG
-    assert int8(16, A.BF16, A.PASS_INT8_PIPELINED) in (A.ERR_CUDA, A.ERR_ARG)
-    assert "pipelined" not in A.last_error()
 
 
 def test_empty_round_needs_no_device(lib):
@@ -361,7 +356,6 @@ def test_binding_constants_match_the_header():
         "ALOCO_PASS_AUTO": A.PASS_AUTO, "ALOCO_PASS_REGISTERS": A.PASS_REGISTERS,
         "ALOCO_PASS_BULK_COPY": A.PASS_BULK_COPY, "ALOCO_PASS_INT8_SPLIT": A.PASS_INT8_SPLIT,
         "ALOCO_PASS_INT8_FUSED": A.PASS_INT8_FUSED, "ALOCO_PASS_TILE": A.PASS_TILE,
-        "ALOCO_PASS_INT8_PIPELINED": A.PASS_INT8_PIPELINED,
         "ALOCO_WAIT_SPIN": A.WAIT_SPIN, "ALOCO_WAIT_BLOCK": A.WAIT_BLOCK,
         "ALOCO_CORR_FULL": A.CORR_FULL, "ALOCO_CORR_MOMENTUM_ONLY": A.CORR_MOMENTUM_ONLY,
         "ALOCO_CORR_NONE": A.CORR_NONE,

@@ -33,8 +33,7 @@ pytestmark = pytest.mark.gpu
 N = 1_000_003
 PLAIN = {"registers": A.PASS_REGISTERS, "bulk_copy": A.PASS_BULK_COPY,
          "tile": A.PASS_TILE}
-INT8 = {"int8_split": A.PASS_INT8_SPLIT, "int8_fused": A.PASS_INT8_FUSED,
-        "int8_pipelined": A.PASS_INT8_PIPELINED}
+INT8 = {"int8_split": A.PASS_INT8_SPLIT, "int8_fused": A.PASS_INT8_FUSED}
 INT8_PARTS = [3 * 4096 + 64, 768, 5001, 12, 4096, N - (3 * 4096 + 64 + 768 +
                                                        5001 + 12 + 4096)]
 
@@ -115,8 +114,6 @@ def test_plain_round_degenerate_cases(case, pass_name, dt, M):
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
 @pytest.mark.parametrize("M", [1, 4, 8, 16])
 def test_int8_round_degenerate_cases(case, form, dt, M):
-    if form == "int8_pipelined" and (dt != "bf16" or M < 2):
-        pytest.skip("the pipelined form takes bf16 replicas and M >= 2")
     w = W.small(N, M, dt, seed=95 + M)
     g, v, xs = _state(w, case)
     g_in, v_in = g.clone(), v.clone()

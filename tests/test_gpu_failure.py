@@ -166,38 +166,3 @@ def test_stalled_int8_worker_group_block_is_reported_and_the_device_stays_usable
     for a_, b_ in zip(x1, x2):
         assert torch.equal(a_.view(torch.int32), b_.view(torch.int32))
 
-
-@pytest.mark.parametrize("M", [8, 16])
-def test_stalled_int8_pipelined_block_is_reported_and_the_device_stays_usable(M):
-    """The pipelined INT8 round (bf16): a block whose copies never arrive
-    makes every thread's bounded wait on it run out; the round reports the
-    timeout after letting its issued copies land, and the next round equals
-    the split form bit for bit."""
-    w = W.small(1 << 22, M, "bf16", seed=7)
-    kw = _kw(w)
-    piped = lambda: A.default_opts(pass_=A.PASS_INT8_PIPELINED)
-    g, v, xs = gpu_inputs(w)
-    st = A.sync_int8(g, v, xs, opts=piped(), **kw)
-    assert st["status"] == A.OK and st["pass_used"] == A.PASS_INT8_PIPELINED
-    block = 2 * st["grid"] + 7                # the third block of CTA 7
-    assert block < w.numel // 4096
-
-    g, v, xs = gpu_inputs(w)
-    A.test_stall_tile(block)
-    t0 = time.time()
-    st = A.sync_int8(g, v, xs, opts=piped(), raise_on_error=False, **kw)
-    took = time.time() - t0
-    assert st["status"] == A.ERR_CUDA
-    assert "timed out" in A.last_error()
-    assert 1.0 < took < 60.0, took
-    torch.cuda.synchronize()
-
-    g1, v1, x1 = gpu_inputs(w)
-    g2, v2, x2 = gpu_inputs(w)
-    st1 = A.sync_int8(g1, v1, x1, opts=piped(), **kw)
-    st2 = A.sync_int8(g2, v2, x2, opts=A.default_opts(pass_=A.PASS_INT8_SPLIT), **kw)
-    assert st1["status"] == st2["status"] == A.OK
-    assert torch.equal(g1.view(torch.int32), g2.view(torch.int32))
-    assert torch.equal(v1.view(torch.int32), v2.view(torch.int32))
-    for a_, b_ in zip(x1, x2):
-        assert torch.equal(a_.view(torch.int16), b_.view(torch.int16))

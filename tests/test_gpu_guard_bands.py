@@ -34,14 +34,11 @@ def _kw(w):
 
 
 @pytest.mark.parametrize("pad", [64, 1])
-@pytest.mark.parametrize("form", [A.PASS_INT8_FUSED, A.PASS_INT8_SPLIT,
-                                  A.PASS_INT8_PIPELINED],
-                         ids=["fused", "split", "pipelined"])
+@pytest.mark.parametrize("form", [A.PASS_INT8_FUSED, A.PASS_INT8_SPLIT],
+                         ids=["fused", "split"])
 @pytest.mark.parametrize("dt,M", [("f32", 3), ("bf16", 8), ("f32", 8), ("bf16", 5),
                                   ("bf16", 16)])
 def test_int8_round(dt, M, form, pad):
-    if form == A.PASS_INT8_PIPELINED and dt != "bf16":
-        pytest.skip("the pipelined form takes bf16 replicas")
     N = sum(PARTS)
     w = W.small(N, M, dt, seed=31)
     g, v, xs = gpu_inputs(w)

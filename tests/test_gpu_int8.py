@@ -97,13 +97,7 @@ def _fits_fused(dt, M):
     return M <= 16
 
 
-FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED,
-         "pipelined": A.PASS_INT8_PIPELINED}
-
-
-def _form_applies(form, dt, M):
-    """The pipelined form takes bf16 replicas and 2 <= M <= 16."""
-    return form != "pipelined" or (dt == "bf16" and 2 <= M <= 16)
+FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
 
 
 @pytest.mark.parametrize("form", sorted(FORMS))
@@ -113,8 +107,6 @@ def _form_applies(form, dt, M):
 def test_int8_round_matches_oracle(dt, M, parts_name, form):
     if form == "fused" and not _fits_fused(dt, M):
         pytest.skip("the fused form holds M <= 16")
-    if not _form_applies(form, dt, M):
-        pytest.skip("the pipelined form takes bf16 replicas and M >= 2")
     parts = PARTS[parts_name]
     N = sum(parts) if parts else 5 * 4096 + 333
     w = W.small(N, M, dt, seed=40 + M)
@@ -143,8 +135,6 @@ def test_int8_forms_agree_bit_for_bit(dt, M):
     sa, _ = schedule_pair(w.schedule)
     out = {}
     for form, p in FORMS.items():
-        if not _form_applies(form, dt, M):
-            continue
         g, v, xs = gpu_inputs(w)
         v.normal_(0, 1e-3, generator=torch.Generator("cuda").manual_seed(M))
         st = A.sync_int8(g, v, xs, parts=parts, H_sel=w.H_sel[0],
@@ -160,15 +150,6 @@ def test_int8_forms_agree_bit_for_bit(dt, M):
     for key in ("D", "C", "mean_sq_norm"):
         assert s1[key] == pytest.approx(s2[key], rel=RTOL_STAT), key
     assert s1["nonfinite"] == s2["nonfinite"] == 0
-    if "pipelined" in out:
-        s3, g3, v3, x3 = out["pipelined"]
-        assert s3["pass_used"] == A.PASS_INT8_PIPELINED
-        assert torch.equal(g3.view(torch.int32), g2.view(torch.int32))
-        assert torch.equal(v3.view(torch.int32), v2.view(torch.int32))
-        for a, b in zip(x3, x2):
-            assert torch.equal(a, b)
-        for key in ("D", "C", "mean_sq_norm"):
-            assert s3[key] == pytest.approx(s2[key], rel=RTOL_STAT), key
 
 
 def test_int8_auto_form():
