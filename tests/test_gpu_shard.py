@@ -228,3 +228,27 @@ def test_unknown_wait_mode_is_rejected():
     st = A.sync(g, v, xs, **_kw(w, A.default_opts(wait=7)),
                 raise_on_error=False)
     assert st["status"] == A.ERR_ARG and "wait" in A.last_error()
+
+
+def test_bench_shard_mode_matches_the_unsharded_round(capsys):
+    """bench.py --shards 3 on one GPU: three shards in sequence and the
+    combine, one timed round; its D_t and C_t equal the unsharded round's on
+    the same seeded inputs within the statistics tolerance."""
+    import json
+    import bench
+    # four 2^24-element generator chunks: three non-empty shards
+    name = "flat50343000_m4_bf16"
+    assert bench.main(["--shards", "3", "--workload", name, "--steps", "1",
+                       "--warmup", "0"]) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["status_ok"] and line["scaling"] == "strong"
+    assert sum(line["config"]["shard_elems"]) == 50_343_000
+    assert all(n > 0 for n in line["config"]["shard_elems"])
+    w = bench.parse_flat(name)
+    g, v, xs = gpu_inputs(w)
+    step, hsel = W.steps_of_rounds(w, 1)[0]
+    sa, _ = schedule_pair(w.schedule)
+    st = A.sync(g, v, xs, H_sel=hsel, H_base=w.H_base, step=step, schedule=sa,
+                outer_lr=w.outer_lr, outer_beta=w.outer_beta)
+    assert_rel(line["D_last"], st["D"], "D", RTOL_STAT)
+    assert_rel(line["C_last"], st["C"], "C", RTOL_STAT)

@@ -169,3 +169,25 @@ def test_noalloc_refuses_a_capturing_stream():
     assert "capture" in A.last_error()
     graph.replay()
     torch.cuda.synchronize()
+
+
+def test_noalloc_caps_a_large_blocks_per_sm_at_occupancy():
+    """blocks_per_sm asks for a residency; every pass caps it at what the
+    kernel's occupancy allows (at most 8 blocks of 256 threads per SM), so
+    even an oversized request stays within the static scratch and gives the
+    allocating entry point's grid, outputs and statistics."""
+    w = W.small(3_000_017, 4, "f32", seed=35)
+    opts = A.default_opts(pass_=A.PASS_REGISTERS, blocks_per_sm=64)
+    out = {}
+    for noalloc in (True, False):
+        g, v, xs = gpu_inputs(w)
+        st = _round(w, g, v, xs, noalloc=noalloc, opts=opts)
+        assert st["status"] == A.OK
+        out[noalloc] = (st, [g, v, *xs])
+    (s1, t1), (s0, t0) = out[True], out[False]
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    assert s1["grid"] == s0["grid"] <= 8 * sms
+    for a, b in zip(t1, t0):
+        assert torch.equal(_bits(a), _bits(b))
+    for k in ("D", "C", "mean_sq_norm", "drift"):
+        assert s1[k] == s0[k], k
