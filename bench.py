@@ -48,6 +48,7 @@ NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 PASSES = {"auto": 0, "registers": 1, "bulk_copy": 2, "int8_split": 3,
           "int8_fused": 4, "tile": 5}
+WAITS = {"spin": 0, "block": 1}
 
 
 def workloads_by_name():
@@ -551,7 +552,8 @@ def run_cuda(args, w):
                                         "sample": f"the same {n} parameters "
                                                   f"on one thread ({t1:.1f} s)"}}
 
-    opts = A.default_opts(time_kernel=1, pass_=PASSES[args.pass_])
+    opts = A.default_opts(time_kernel=1, pass_=PASSES[args.pass_],
+                          wait=WAITS[args.wait])
     parts = W.tensor_sizes(w)
     step_ms, kern_ms, statuses = [], [], []
     ev = [(torch.cuda.Event(enable_timing=True),
@@ -635,7 +637,7 @@ def run_cuda(args, w):
             "data": "synthetic (seeded; Llama-shaped parameter set, "
                     "shared/private drift noise)",
             "config": dict(config_block(w), comm=args.comm,
-                           l2=l2_note(w, l2)),
+                           l2=l2_note(w, l2), wait=args.wait),
             "rounds_per_s_per_gpu": 1e3 / ms_step,
             "elem_per_s": value * w.numel * w.M,
             "kernel_ms": ms_kern, "kernel_ms_stat": "median",
@@ -753,10 +755,10 @@ def run_shard(args, w):
     GPU.  Under torchrun: rank r holds and runs shard r of WORLD_SIZE shards,
     and the ranks all-gather their partials (one small struct each) over
     NCCL before combining them, so every rank obtains the same D_t and C_t.
-    A step is one whole round (every shard, the exchange and the combine),
-    timed on the host around calls that return once their kernels are done;
-    the value is whole rounds per second (total work fixed as ranks are
-    added: strong scaling)."""
+    A step is one whole round: every shard this rank holds and the exchange,
+    timed with CUDA events on the launch stream (the all-gather is enqueued
+    on it), then the host combine; the value is whole rounds per second
+    (total work fixed as ranks are added: strong scaling)."""
     import torch
     from paper_2609_36662_gb300 import aloco as A
     from paper_2609_36662_gb300 import workloads as W
@@ -784,8 +786,9 @@ def run_shard(args, w):
     sched = A.Schedule.make(s.kind, s.peak_lr, s.final_lr, s.warmup_steps,
                             s.total_steps)
     stream = torch.cuda.Stream(device)
-    opts = A.default_opts(time_kernel=1, pass_=PASSES[args.pass_])
-    step_ms, kern_ms, statuses, D, C = [], [], [], [], []
+    opts = A.default_opts(time_kernel=1, pass_=PASSES[args.pass_],
+                          wait=WAITS[args.wait])
+    step_ms, host_ms, kern_ms, statuses, D, C = [], [], [], [], [], []
 
     def one_round(k):
         step, hsel = rounds[k]
@@ -796,7 +799,10 @@ def run_shard(args, w):
         stream.synchronize()
         if world > 1:
             torch.distributed.barrier()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
         t0 = time.perf_counter()
+        e0.record(stream)
         blobs, ms = [], 0.0
         for _, _, g, v, xs in pieces:
             rc, part = A.sync_shard(g, v, xs, H_sel=hsel, H_base=w.H_base,
@@ -807,18 +813,22 @@ def run_shard(args, w):
             blobs.append(part.to_bytes())
             ms += max(part.kernel_ms, 0.0)
         if world > 1:
-            blobs = gather_partials(blobs[0], world, device)
+            with torch.cuda.stream(stream):
+                blobs = gather_partials(blobs[0], world, device)
+        e1.record(stream)
+        e1.synchronize()
         st = A.combine_partials([A.Partials.from_bytes(b) for b in blobs])
         t1 = time.perf_counter()
-        return (t1 - t0) * 1e3, ms, st
+        return e0.elapsed_time(e1), (t1 - t0) * 1e3, ms, st
 
     for k in range(args.warmup):
         one_round(k)
     torch.cuda.synchronize()
     with ClockSampler(device.index) as clocks:
         for k in range(args.warmup, args.warmup + args.steps):
-            t, ms, st = one_round(k)
+            t, th, ms, st = one_round(k)
             step_ms.append(t)
+            host_ms.append(th)
             kern_ms.append(ms)
             statuses.append(st["status"])
             D.append(st["D"])
@@ -838,6 +848,7 @@ def run_shard(args, w):
             "metric": METRIC, "value": 1e3 / ms_step, "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": ms_step, "ms_per_step_stat": "median",
+            "ms_per_step_host": statistics.median(host_ms),
             "higher_is_better": True, "scaling": "strong",
             "vs_baseline": None, "dtype": "f32", "replica_dtype": w.dtype,
             "data": "synthetic (seeded; Llama-shaped parameter set, "
@@ -1224,6 +1235,10 @@ def main(argv=None):
                    default="computed",
                    help="--mode adamw: compute the clipping norms (two "
                         "passes) or take them from the caller (one pass)")
+    p.add_argument("--wait", choices=sorted(WAITS), default="spin",
+                   help="how the round call waits for its kernel: poll the "
+                        "published statistics (spin) or sleep on a "
+                        "blocking-sync event (block)")
     p.add_argument("--shards", type=int, default=0,
                    help="run the round as shards (aloco_sync_shard + "
                         "aloco_combine_partials): G shards in sequence on "

@@ -4,7 +4,9 @@
 // CTAs of T threads work through 4096-element codec blocks (grid stride),
 // 4096 / T elements per thread in chunks of 4 (chunk c of thread t at
 // 4t + c x 4T, so warp accesses to shared memory are contiguous): two
-// 512-thread CTAs per SM where they fit, else one 1024-thread CTA (see
+// 512-thread CTAs per SM where they fit (where only the staging of theta
+// and v keeps them from fitting, each thread reads its theta and v from
+// global memory instead; see direct_gv), else one 1024-thread CTA (see
 // fused_threads).  Per block:
 //   1. theta, v and the M replica slices arrive in shared memory by bulk
 //      copies (cp.async.bulk, one per array, issued by thread 0 and
@@ -79,12 +81,6 @@ __host__ __device__ constexpr int fused_group() {
     if (M <= 8 || BF16) return M;
     return balanced_group(M, 3);
 }
-// theta, v (fp32) and one group's replica slices of one block
-template <int M, bool BF16>
-__host__ __device__ constexpr size_t in_bytes() {
-    return (size_t)kI8Block * (8 + fused_group<M, BF16>() * esize<BF16>());
-}
-
 // the static shared arrays of the kernel and of the final reduction (an
 // upper bound)
 template <int M, int T>
@@ -95,6 +91,46 @@ __host__ __device__ constexpr size_t static_bytes() {
 template <int C>
 __host__ __device__ constexpr size_t cta_budget() {
     return C == 1 ? kSmemPerCta : kSmemPerSm / C - kSmemReserved;
+}
+// Two 512-thread CTAs per SM with theta and v staged beside the replicas
+// (and the replica-type output tile), or with theta and v read by every
+// thread straight from global memory instead.
+template <int M, bool BF16>
+__host__ __device__ constexpr bool fits_two_staged() {
+    return (size_t)kI8Block * (8 + fused_group<M, BF16>() * esize<BF16>()) +
+               (size_t)kI8Block * esize<BF16>() + static_bytes<M, 512>() <=
+           cta_budget<2>();
+}
+template <int M, bool BF16>
+__host__ __device__ constexpr bool fits_two_direct() {
+    return (size_t)kI8Block * (fused_group<M, BF16>() * esize<BF16>()) +
+               (size_t)kI8Block * esize<BF16>() + static_bytes<M, 512>() <=
+           cta_budget<2>();
+}
+// theta and v are not staged where that alone keeps two CTAs per SM from
+// fitting (bf16 M = 9..12, fp32 M = 4, 5): each thread loads its own theta
+// (before its wait for the replicas) and v from global memory, the same
+// bytes read once, and the shared memory holds the replicas only.
+// Measured on GB300 (4e8 parameters, fraction of the copy peak), against
+// one 1024-thread CTA with theta and v staged: bf16 M = 9 0.860 (0.726),
+// M = 10 0.879 (0.738), M = 12 0.835 (0.737); fp32 M = 4 0.939 (0.903),
+// M = 5 0.926 (0.930).  bf16 M >= 13 does not fit two CTAs even so (its
+// replicas alone take more than half an SM).  ALOCO_I8_DIRECT = 0 turns it
+// off (a tuning knob).
+#ifndef ALOCO_I8_DIRECT
+#define ALOCO_I8_DIRECT 1
+#endif
+template <int M, bool BF16>
+__host__ __device__ constexpr bool direct_gv() {
+    return ALOCO_I8_DIRECT && fused_group<M, BF16>() == M && !fits_two_staged<M, BF16>() &&
+           fits_two_direct<M, BF16>();
+}
+// theta, v (fp32, unless read directly) and one group's replica slices of
+// one block
+template <int M, bool BF16>
+__host__ __device__ constexpr size_t in_bytes() {
+    return (size_t)kI8Block *
+           ((direct_gv<M, BF16>() ? 0 : 8) + fused_group<M, BF16>() * esize<BF16>());
 }
 // The fp32 theta' and v' tiles fit beside the input and the replica tile.
 template <int M, bool BF16, int T, int C>
@@ -254,6 +290,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     constexpr int NG = (M + G - 1) / G;          // groups per block
     constexpr bool GROUPED = NG > 1;
     constexpr int EA = GROUPED ? G : M;          // energy accumulators a thread
+    constexpr bool DGV = direct_gv<M, BF16>();   // theta, v read from global memory
     constexpr uint32_t kGVBytes = kI8Block * 4;  // one fp32 array of a block
     constexpr uint32_t kXBytes = kI8Block * ES;  // one replica slice
     // Single buffers suffice: red_w is read between a group's first barrier
@@ -265,9 +302,9 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     __shared__ __align__(16) float2 sr[W][G + (G & 1)];  // per warp: (scale, 1/scale)
     __shared__ __align__(8) unsigned long long full_bar;
     extern __shared__ __align__(128) unsigned char smem[];
-    float *sg = reinterpret_cast<float *>(smem);
-    float *sv = sg + kI8Block;
-    unsigned char *sx = smem + 2 * kGVBytes;
+    float *sg = reinterpret_cast<float *>(smem);  // theta (staged only if !DGV)
+    float *sv = sg + kI8Block;                      // v (staged only if !DGV)
+    unsigned char *sx = smem + (DGV ? 0 : 2 * kGVBytes);
     unsigned char *ox = sx + G * kXBytes;             // theta' in the replica type
     float *og = BF16 ? reinterpret_cast<float *>(ox + kXBytes)  // theta' (fp32)
                      : reinterpret_cast<float *>(ox);
@@ -311,6 +348,21 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     // thread t holds the 4-element chunks at 4t + c x 4T (c < PER / 4), so
     // every warp access to a staged array is contiguous
     auto el = [&](int i) { return (i >> 2) * (4 * T) + 4 * t + (i & 3); };
+    // a thread's elements of an fp32 array read straight from global memory:
+    // 16-byte streaming loads on whole aligned blocks, element loads (0
+    // beyond the block's end) otherwise
+    auto load_direct = [&](float (&o)[PER], const float *src, int64_t s, int l, bool whole) {
+#pragma unroll
+        for (int c = 0; c < PER; c += 4) {
+            if (whole) {
+                const float4 q = __ldcs(reinterpret_cast<const float4 *>(src + s + el(c)));
+                o[c] = q.x; o[c + 1] = q.y; o[c + 2] = q.z; o[c + 3] = q.w;
+            } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) o[c + i] = el(c + i) < l ? src[s + el(c + i)] : 0.f;
+            }
+        }
+    };
 
     // whole blocks at 16-byte aligned addresses move by bulk copies
     auto bulk_block = [&](int64_t s, int l) {
@@ -324,8 +376,8 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
             return;  // testing only: this phase never completes
         const int m0 = q * G;
         const int gq = M - m0 < G ? M - m0 : G;
-        mbar_arrive_expect_tx(bar, (q == 0 ? 2 * kGVBytes : 0) + gq * kXBytes);
-        if (q == 0) {
+        mbar_arrive_expect_tx(bar, (q == 0 && !DGV ? 2 * kGVBytes : 0) + gq * kXBytes);
+        if (q == 0 && !DGV) {
             bulk_load(smem_addr(sg), a.g + s, kGVBytes, bar);
             bulk_load(smem_addr(sv), a.v + s, kGVBytes, bar);
         }
@@ -345,7 +397,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         for (int i = 0; i < PER; ++i) {
             const int e = el(i);
             const bool in = e < l;
-            if (q == 0) {
+            if (q == 0 && !DGV) {
                 sg[e] = in ? a.g[s + e] : 0.f;
                 sv[e] = in ? a.v[s + e] : 0.f;
             }
@@ -403,6 +455,11 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         float2 g2[NP];    // theta, as pairs
         float2 sum2[NP];  // the workers' decoded sum
         if constexpr (!GROUPED) {
+            if constexpr (DGV) {
+                // theta straight from global memory, issued before the wait
+                // for the replicas so the two overlap
+                load_direct(g, a.g, start, len, bulk);
+            }
             bool timed_out = false;
             if (bulk) {
                 timed_out = !mbar_wait(bar, phase, nullptr);
@@ -410,10 +467,12 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
                 phase ^= 1;
             }
 
+            if constexpr (!DGV) {
 #pragma unroll
-            for (int c = 0; c < PER; c += 4) {
-                const float4 q = *reinterpret_cast<const float4 *>(sg + el(c));
-                g[c] = q.x; g[c + 1] = q.y; g[c + 2] = q.z; g[c + 3] = q.w;
+                for (int c = 0; c < PER; c += 4) {
+                    const float4 q = *reinterpret_cast<const float4 *>(sg + el(c));
+                    g[c] = q.x; g[c + 1] = q.y; g[c + 2] = q.z; g[c + 3] = q.w;
+                }
             }
 #pragma unroll
             for (int j = 0; j < NP; ++j) g2[j] = make_float2(g[2 * j], g[2 * j + 1]);
@@ -678,10 +737,14 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         }
         // 4. the mean's codec
         float v[PER];
+        if constexpr (DGV) {
+            load_direct(v, a.v, start, len, bulk);
+        } else {
 #pragma unroll
-        for (int c = 0; c < PER; c += 4) {
-            const float4 q = *reinterpret_cast<const float4 *>(sv + el(c));
-            v[c] = q.x; v[c + 1] = q.y; v[c + 2] = q.z; v[c + 3] = q.w;
+            for (int c = 0; c < PER; c += 4) {
+                const float4 q = *reinterpret_cast<const float4 *>(sv + el(c));
+                v[c] = q.x; v[c + 1] = q.y; v[c + 2] = q.z; v[c + 3] = q.w;
+            }
         }
         float sum[PER];
 #pragma unroll
