@@ -108,22 +108,25 @@ __host__ __device__ constexpr bool fits_two_direct() {
            cta_budget<2>();
 }
 // theta and v are not staged where that alone keeps two CTAs per SM from
-// fitting (bf16 M = 9..12, fp32 M = 4, 5): each thread loads its own theta
-// (before its wait for the replicas) and v from global memory, the same
-// bytes read once, and the shared memory holds the replicas only.
-// Measured on GB300 (4e8 parameters, fraction of the copy peak), against
-// one 1024-thread CTA with theta and v staged: bf16 M = 9 0.860 (0.726),
-// M = 10 0.879 (0.738), M = 12 0.835 (0.737); fp32 M = 4 0.939 (0.903),
-// M = 5 0.926 (0.930).  bf16 M >= 13 does not fit two CTAs even so (its
-// replicas alone take more than half an SM).  ALOCO_I8_DIRECT = 0 turns it
-// off (a tuning knob).
+// fitting (bf16 M = 9..12, fp32 M = 4, 5), nor for fp32 M = 2, 3: each
+// thread loads its own theta (before its wait for the replicas) and v from
+// global memory, the same bytes read once, and the shared memory holds the
+// replicas only.  Measured on GB300 (4e8 parameters, fraction of the copy
+// peak; in brackets with theta and v staged, on one 1024-thread CTA where
+// two do not fit): bf16 M = 9 0.860 (0.726), M = 10 0.879 (0.738), M = 12
+// 0.835 (0.737); fp32 M = 2 0.979 (0.965), M = 3 0.959 (0.921), M = 4
+// 0.939 (0.903), M = 5 0.926 (0.930).  Staging stays faster for fp32 M = 1
+// (0.984 against 0.931) and bf16 M <= 8 (M = 8: 0.915 against 0.839).
+// bf16 M >= 13 does not fit two CTAs even so (its replicas alone take more
+// than half an SM).  ALOCO_I8_DIRECT = 0 turns it off, 2 takes it wherever
+// two CTAs fit (tuning knobs).
 #ifndef ALOCO_I8_DIRECT
 #define ALOCO_I8_DIRECT 1
 #endif
 template <int M, bool BF16>
 __host__ __device__ constexpr bool direct_gv() {
-    return ALOCO_I8_DIRECT && fused_group<M, BF16>() == M && !fits_two_staged<M, BF16>() &&
-           fits_two_direct<M, BF16>();
+    return ALOCO_I8_DIRECT && fused_group<M, BF16>() == M && fits_two_direct<M, BF16>() &&
+           (ALOCO_I8_DIRECT == 2 || !fits_two_staged<M, BF16>() || (!BF16 && M >= 2));
 }
 // theta, v (fp32, unless read directly) and one group's replica slices of
 // one block
