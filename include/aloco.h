@@ -124,10 +124,10 @@ typedef enum {
  * The INT8-communicated round (aloco_sync_int8) has two forms of its own:
  *   INT8_SPLIT a block-scale kernel, then an apply kernel that reads the
  *              replicas again (any M <= 16);
- *   INT8_FUSED one kernel that stages each block of theta, v and the
- *              replicas in shared memory, reading every replica once
- *              (any M <= 16; above 8 fp32 replicas it stages each
- *              block's replicas in groups);
+ *   INT8_FUSED one kernel that stages each block of the replicas (and of
+ *              theta and v, for the shapes where that measured faster) in
+ *              shared memory, reading every array once (any M <= 16; above
+ *              8 fp32 replicas it stages each block's replicas in groups);
  *   AUTO       the form measured faster on GB300 for (M, dtype).
  * The two INT8 forms give the same theta', v' and replicas bit for bit.
  * aloco_sync / aloco_sync_ex reject the INT8 values and aloco_sync_int8 the
