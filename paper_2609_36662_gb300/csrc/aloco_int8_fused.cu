@@ -68,17 +68,35 @@ __host__ __device__ constexpr int esize() { return BF16 ? 2 : 4; }
 __host__ __device__ constexpr int balanced_group(int M, int cap) {
     return (M + (M + cap - 1) / cap - 1) / ((M + cap - 1) / cap);
 }
-// All M for M <= 8.  Above, groups of 3 for fp32: two 512-thread CTAs per
-// SM then fit, and measured 0.84-0.94 of the copy peak for M = 9..16
-// against 0.54-0.60 for groups of 8 on one 1024-thread CTA (the split form:
-// 0.66-0.67).  ALOCO_I8_FUSED_G caps the group (a tuning knob).
+// All M for M <= 8.  Above, fp32 stages the replicas in groups on two
+// 512-thread CTAs per SM: of up to 5 workers with theta and v read directly
+// (grouped_direct), else of 3 with theta and v staged (0.84-0.94 of the
+// copy peak for M = 9..16 against 0.54-0.60 for groups of 8 on one
+// 1024-thread CTA; the split form: 0.66-0.67).  ALOCO_I8_FUSED_G caps the
+// group (a tuning knob).
 #ifndef ALOCO_I8_FUSED_G
 #define ALOCO_I8_FUSED_G 0
 #endif
+// fp32 with M > 8: theta and v read directly from global memory, which
+// leaves room for groups of up to 5 workers on two 512-thread CTAs per SM
+// (a 16-worker block in 4 groups instead of 6).  Measured on GB300 (4e8
+// parameters, fraction of the copy peak) against groups of 3 with theta and
+// v staged: M = 9 0.949 (0.904), M = 12 0.878 (0.867), M = 16 0.869
+// (0.808); groups of at most 4 gave 0.865, 0.880 and 0.869.
+// ALOCO_I8_GDIRECT sets the group cap (0: groups of 3 with theta and v
+// staged; a tuning knob).
+#ifndef ALOCO_I8_GDIRECT
+#define ALOCO_I8_GDIRECT 5
+#endif
+template <int M, bool BF16>
+__host__ __device__ constexpr bool grouped_direct() {
+    return ALOCO_I8_GDIRECT > 0 && !BF16 && M > 8 && ALOCO_I8_FUSED_G == 0;
+}
 template <int M, bool BF16>
 __host__ __device__ constexpr int fused_group() {
     if (ALOCO_I8_FUSED_G) return balanced_group(M, ALOCO_I8_FUSED_G);
     if (M <= 8 || BF16) return M;
+    if (grouped_direct<M, BF16>()) return balanced_group(M, ALOCO_I8_GDIRECT);
     return balanced_group(M, 3);
 }
 // the static shared arrays of the kernel and of the final reduction (an
@@ -125,6 +143,7 @@ __host__ __device__ constexpr bool fits_two_direct() {
 #endif
 template <int M, bool BF16>
 __host__ __device__ constexpr bool direct_gv() {
+    if (grouped_direct<M, BF16>()) return true;
     return ALOCO_I8_DIRECT && fused_group<M, BF16>() == M && fits_two_direct<M, BF16>() &&
            (ALOCO_I8_DIRECT == 2 || !fits_two_staged<M, BF16>() || (!BF16 && M >= 2));
 }
@@ -591,6 +610,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
             for (int q = 0; q < NG; ++q) {
                 const int m0 = q * G;                      // first worker
                 const int GQ = M - m0 < G ? M - m0 : G;    // workers in the group
+                if (DGV && q == 0) load_direct(g, a.g, start, len, bulk);
                 bool timed_out = false;
                 if (bulk) {
                     timed_out = !mbar_wait(bar, phase, nullptr);
@@ -598,10 +618,12 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
                     phase ^= 1;
                 }
                 if (q == 0) {
+                    if constexpr (!DGV) {
 #pragma unroll
-                    for (int c = 0; c < PER; c += 4) {
-                        const float4 v4 = *reinterpret_cast<const float4 *>(sg + el(c));
-                        g[c] = v4.x; g[c + 1] = v4.y; g[c + 2] = v4.z; g[c + 3] = v4.w;
+                        for (int c = 0; c < PER; c += 4) {
+                            const float4 v4 = *reinterpret_cast<const float4 *>(sg + el(c));
+                            g[c] = v4.x; g[c + 1] = v4.y; g[c + 2] = v4.z; g[c + 3] = v4.w;
+                        }
                     }
 #pragma unroll
                     for (int j = 0; j < NP; ++j) g2[j] = make_float2(g[2 * j], g[2 * j + 1]);
