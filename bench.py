@@ -123,13 +123,24 @@ def host_memory():
     return out
 
 
-def pinned_budget(mem) -> int:
-    """Pinned host bytes the e2e leg may take: half of what is available
-    (and of the cgroup limit), so the host keeps room for the rest."""
+def pinned_budget(mem, ranks_on_host: int = 1) -> int:
+    """Pinned host bytes one rank's e2e leg may take: half of what is
+    available (and of the cgroup limit), shared by the ranks on this host,
+    so the host keeps room for the rest."""
     cands = [v for v in (mem.get("mem_available_bytes"),
                          mem.get("cgroup_limit_bytes"),
                          mem.get("host_ram_bytes")) if v]
-    return int(0.5 * min(cands)) if cands else 0
+    if not cands:
+        return 0
+    return int(0.5 * min(cands) / max(1, ranks_on_host))
+
+
+def ranks_on_host() -> int:
+    """Ranks of this job on this host (torchrun's LOCAL_WORLD_SIZE)."""
+    try:
+        return max(1, int(os.environ.get("LOCAL_WORLD_SIZE", "1")))
+    except ValueError:
+        return 1
 
 
 def hbm_peak():
@@ -682,13 +693,19 @@ def run_e2e(args, w, g, v, xs, sched, stream, rounds, world, device,
     # into theta, v); the INT8 leg copies theta', v' out to two more arrays
     pinned = h2d + (d2h if int8_parts is not None else 0)
     mem = host_memory()
-    budget = pinned_budget(mem)
-    if budget and pinned > budget:
+    local = ranks_on_host()
+    budget = pinned_budget(mem, local)
+    # every rank decides the same way, so all take the e2e leg or none do
+    skip = 1.0 if (budget and pinned > budget) else 0.0
+    if world > 1:
+        skip = reduce_max(skip, world, device)
+    if skip:
         return {"value": None, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "pinned_bytes": pinned, **mem,
-                "skipped": f"the pinned host state ({pinned / 1e9:.1f} GB) "
-                           f"exceeds half of the host memory available "
-                           f"({budget / 1e9:.1f} GB allowed)"}
+                "ranks_on_host": local,
+                "skipped": f"the pinned host state ({pinned / 1e9:.1f} GB per "
+                           f"rank) exceeds this rank's share of half of the "
+                           f"host memory available ({budget / 1e9:.1f} GB)"}
     t_pin = time.perf_counter()
     hg = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)
     hv = torch.empty(w.numel, dtype=torch.float32, pin_memory=True)

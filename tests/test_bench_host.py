@@ -76,3 +76,14 @@ def test_recorded_entries_follow_the_kernel_source(tmp_path, monkeypatch):
     monkeypatch.setattr(bench, "kernel_source_hash", lambda k: "changed")
     assert bench.recorded_traffic("w", "k") is None
     assert bench.recorded_occupancy("w", "k") is None
+
+
+def test_pinned_budget_is_shared_by_the_ranks_on_a_host():
+    import bench
+    mem = {"host_ram_bytes": 200e9, "mem_available_bytes": 180e9,
+           "cgroup_limit_bytes": None}
+    assert bench.pinned_budget(mem) == int(90e9)
+    assert bench.pinned_budget(mem, 8) == int(90e9 / 8)
+    mem["cgroup_limit_bytes"] = 100e9
+    assert bench.pinned_budget(mem, 2) == int(25e9)
+    assert bench.pinned_budget({}, 4) == 0
