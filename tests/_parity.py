@@ -458,3 +458,72 @@ def compare_whole_vector(w: W.Workload, g_in, v_in, x_in, g, v, xs, corr,
                    go, s)
     return {"theta_candidates": fg.check(), "v_candidates": fv.check(),
             "replica_candidates": fx.check()}
+
+
+def int8_slices(parts, slice_elems=1 << 24):
+    """(start, length) slices of a vector made of tensor parts, each inside
+    one part and starting at a multiple of 4096 from that part's start, so
+    every slice holds whole codec blocks (they restart at every part)."""
+    step = max(4096, slice_elems // 4096 * 4096)
+    out, off = [], 0
+    for p in parts:
+        for o in range(0, p, step):
+            out.append((off + o, min(step, p - o)))
+        off += p
+    return out
+
+
+def compare_int8_whole_vector(w: W.Workload, parts, g_in, v_in, x_in, g, v, xs,
+                              corr, eps=1e-8, slice_elems=1 << 24, threads=16):
+    """The INT8-communicated round against the oracle over the WHOLE vector:
+    slice by slice (whole codec blocks each), the oracle's INT8 round runs on
+    host copies of the device snapshot in threads, and every element of
+    theta', v' and replica 0 is held to the tolerances of compare_round; the
+    slices' drift energies and squared decoded aggregates are added in slice
+    order into the whole round's statistics, which are returned (D from the
+    pre-quantisation pseudo-gradients, C from the decoded aggregate)."""
+    dt = O.F32 if w.dtype == "f32" else O.BF16
+    fg, fv, fx = (_FieldCheck("theta'"), _FieldCheck("v'"),
+                  _FieldCheck("replica 0"))
+    E = [0.0] * w.M
+    B = 0.0
+    slices = int8_slices(parts, slice_elems)
+
+    def work(s, n, gh, vh, xh):
+        return O.int8_round(gh, vh, xh, dt, [n], corr.mu_t, corr.eta_out,
+                            corr.inv_norm, eps)
+
+    def check(s, n, r):
+        nonlocal B
+        e = s + n
+        fg.add(_abs_diff(g[s:e].cpu().numpy(), r["g"]), r["g"], s)
+        fv.add(_abs_diff(v[s:e].cpu().numpy(), r["v"]), r["v"], s)
+        x0 = to_numpy_bits(xs[0][s:e])
+        if dt == O.F32:
+            fx.add(_abs_diff(x0, r["x"][0]), r["x"][0], s)
+        else:
+            ov = O.bf16_bits_to_float(r["x"][0])
+            fx.add(_abs_diff(O.bf16_bits_to_float(x0), ov) - bf16_ulp(ov),
+                   r["g"], s)
+        for m in range(w.M):
+            E[m] += r["drift"][m]
+        B += r["mean_sq_norm"]
+
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        pending = []
+        for s, n in slices:
+            e = s + n
+            fut = ex.submit(work, s, n, g_in[s:e].cpu().numpy(),
+                            v_in[s:e].cpu().numpy(),
+                            [to_numpy_bits(x[s:e]) for x in x_in])
+            pending.append((s, n, fut))
+            if len(pending) >= 2 * threads:
+                s0, n0, f0 = pending.pop(0)
+                check(s0, n0, f0.result())
+        for s0, n0, f0 in pending:
+            check(s0, n0, f0.result())
+    fg.check()
+    fv.check()
+    fx.check()
+    D = sum(E) / w.M
+    return {"D": D, "C": w.M * B / (D + eps), "mean_sq_norm": B, "drift": E}

@@ -10,8 +10,8 @@ from paper_2609_36662_gb300 import aloco as A
 from paper_2609_36662_gb300 import workloads as W
 
 from _parity import (RTOL_STAT, assert_bf16_replica, assert_corr, assert_field,
-                     assert_stats, gpu_inputs, oracle_corr, schedule_pair,
-                     to_numpy_bits)
+                     assert_stats, compare_int8_whole_vector, gpu_inputs,
+                     oracle_corr, schedule_pair, to_numpy_bits)
 
 pytestmark = pytest.mark.gpu
 
@@ -194,9 +194,9 @@ def test_int8_round_with_normalisation_and_nonfinite():
 
 def test_int8_round_full_size_llama150m():
     """The 150M layout (111 tensor parts, 8 fp32 workers) in one INT8 round:
-    sampled whole codec blocks against the oracle, and the full statistics
-    from the oracle over every part (threaded over parts)."""
-    import concurrent.futures as cf
+    every element against the oracle's INT8 round, run slice by slice (whole
+    codec blocks each) on a device snapshot of the inputs, and the full
+    statistics from the slices' sums."""
     w = W.llama_150m()
     parts = W.tensor_sizes(w)
     g, v, xs = gpu_inputs(w)
@@ -210,33 +210,9 @@ def test_int8_round_full_size_llama150m():
                      outer_beta=w.outer_beta)
     assert st["status"] == A.OK
     assert_corr(st["corr"], corr)
-    offs = np.concatenate([[0], np.cumsum(parts)])
-    # full statistics: the oracle over each part on its own thread
-    E = np.zeros((len(parts), w.M))
-    B = np.zeros(len(parts))
-
-    def work(p):
-        s, e = int(offs[p]), int(offs[p + 1])
-        r = O.int8_round(g_in[s:e].cpu().numpy(), v_in[s:e].cpu().numpy(),
-                         [x[s:e].cpu().numpy() for x in x_in], O.F32,
-                         [e - s], corr.mu_t, corr.eta_out, corr.inv_norm)
-        E[p] = r["drift"]
-        B[p] = r["mean_sq_norm"]
-        return p, s, r
-    rng = np.random.default_rng(0)
-    check = set(rng.choice(len(parts), 12, replace=False).tolist()) | {0, 1,
-                                                                      len(parts) - 1}
-    with cf.ThreadPoolExecutor(16) as ex:
-        for p, s, r in ex.map(work, range(len(parts))):
-            if p in check:
-                e = s + r["g"].size
-                assert_field(g[s:e].cpu().numpy(), r["g"], f"theta' part {p}")
-                assert_field(v[s:e].cpu().numpy(), r["v"], f"v' part {p}")
-    Em = [float(E[:, m].sum()) for m in range(w.M)]
-    D = sum(Em) / w.M
-    Bt = float(B.sum())
-    orc = {"D": D, "C": w.M * Bt / (D + 1e-8), "mean_sq_norm": Bt,
-           "drift": Em}
+    gi = g.view(torch.int32)
+    assert all(torch.equal(x.view(torch.int32), gi) for x in xs)
+    orc = compare_int8_whole_vector(w, parts, g_in, v_in, x_in, g, v, xs, corr)
     assert_stats(st, orc, w.M)
 
 
