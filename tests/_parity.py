@@ -51,21 +51,46 @@ def schedule_pair(spec: W.ScheduleSpec):
                        spec.warmup_steps, spec.total_steps))
 
 
-def field_error(gpu: np.ndarray, orc: np.ndarray) -> float:
+def field_error(gpu: np.ndarray, orc: np.ndarray, terms=None) -> float:
+    """Largest error relative to max(|oracle|, rms of the oracle field, and,
+    where given, the magnitude of the terms the value is formed from)."""
     gpu = np.asarray(gpu, np.float64)
     orc = np.asarray(orc, np.float64)
     if orc.size == 0:
         return 0.0
     rms = float(np.sqrt(np.mean(orc * orc)))
     scale = np.maximum(np.abs(orc), max(rms, 1e-300))
+    if terms is not None:
+        scale = np.maximum(scale, np.asarray(terms, np.float64))
     err = np.abs(gpu - orc) / scale
     err[(gpu == orc)] = 0.0
     return float(err.max())
 
 
-def assert_field(gpu, orc, name, rtol=RTOL_FIELD):
-    e = field_error(gpu, orc)
+def assert_field(gpu, orc, name, rtol=RTOL_FIELD, terms=None):
+    e = field_error(gpu, orc, terms)
     assert e <= rtol, f"{name}: max scaled error {e:.3e} > {rtol:.0e}"
+
+
+def step_terms(g, v, xs, dtype, mu_t, eta_out, inv_norm):
+    """Per element, the magnitudes of the terms of the corrected Nesterov
+    step (Eq. autoloco-corrected-nesterov): v' = mu v + Dtil with Dtil =
+    inv_norm S / M, S = sum_m (theta - x_m), and theta' = theta - eta (Dtil +
+    mu v').  Evaluated in fp32, each result carries rounding errors of the
+    size of its terms (S alone rounds M - 1 times), so where the terms
+    cancel (a vector of a few elements has no rms to fall back on) the
+    tolerance scales with them: |mu v| + |inv_norm / M| sum_m |theta - x_m|
+    for v', and |theta| + |eta| (that + mu (that)) for theta'."""
+    g = np.asarray(g, np.float64)
+    v = np.asarray(v, np.float64)
+    a = np.zeros_like(g)
+    for x in xs:
+        xf = (O.bf16_bits_to_float(x) if dtype == O.BF16 else np.asarray(x)).astype(np.float64)
+        a += np.abs(g - xf)
+    dt = abs(inv_norm) / len(xs) * a
+    tv = abs(mu_t) * np.abs(v) + dt
+    tg = np.abs(g) + abs(eta_out) * (dt + abs(mu_t) * tv)
+    return tg, tv
 
 
 def fp32_ulp(values) -> np.ndarray:
@@ -224,8 +249,12 @@ def run_oracle_round(g, v, xs, w: W.Workload, step: int, H_sel: int,
     vh = v.cpu().numpy() if isinstance(v, torch.Tensor) else v
     xh = [to_numpy_bits(x) if isinstance(x, torch.Tensor) else x for x in xs]
     dt = O.F32 if w.dtype == "f32" else O.BF16
-    return O.sync_round(gh, vh, xh, dt, so, step, H_sel, w.H_base, w.outer_lr,
-                        w.outer_beta, eps=eps, normalize=normalize, mode=mode)
+    orc = O.sync_round(gh, vh, xh, dt, so, step, H_sel, w.H_base, w.outer_lr,
+                       w.outer_beta, eps=eps, normalize=normalize, mode=mode)
+    c = orc["corr"]
+    orc["g_terms"], orc["v_terms"] = step_terms(gh, vh, xh, dt, c.mu_t, c.eta_out,
+                                                c.inv_norm)
+    return orc
 
 
 def compare_round(w, st, orc, g, v, xs):
@@ -233,8 +262,8 @@ def compare_round(w, st, orc, g, v, xs):
     assert st["nonfinite"] == orc["nonfinite"]
     assert_corr(st["corr"], orc["corr"])
     assert_stats(st, orc, w.M)
-    assert_field(g.cpu().numpy(), orc["g"], "theta'")
-    assert_field(v.cpu().numpy(), orc["v"], "v'")
+    assert_field(g.cpu().numpy(), orc["g"], "theta'", terms=orc.get("g_terms"))
+    assert_field(v.cpu().numpy(), orc["v"], "v'", terms=orc.get("v_terms"))
     gg = g.cpu().numpy()
     for m, x in enumerate(xs):
         if w.dtype == "f32":

@@ -55,7 +55,7 @@ def test_int8_round(dt, M, form, pad):
 @pytest.mark.parametrize("pad", [64, 1])
 def test_int8_codec(pad):
     N = sum(PARTS)
-    y = torch.randn(N, device="cuda") * 1e-3
+    y = torch.randn(N, device="cuda", generator=torch.Generator("cuda").manual_seed(pad)) * 1e-3
     yb, yi = _padded(y, pad, 5.0)
     nb = A.int8_num_blocks(PARTS)
     cb = torch.full((N + 2 * pad,), 99, dtype=torch.int8, device="cuda")
