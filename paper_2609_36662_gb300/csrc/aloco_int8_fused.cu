@@ -8,6 +8,10 @@
 // and v keeps them from fitting, each thread reads its theta and v from
 // global memory instead; see direct_gv), else one 1024-thread CTA (see
 // fused_threads).  Per block:
+//   0. thread 0 locates the next block and, for some shapes, leaves its
+//      place in shared memory for every thread (see ALOCO_I8_NEXT_SMEM);
+//      where bf16 runs one CTA per SM it also asks L2 to fetch the next
+//      block's arrays (see ALOCO_I8_PREFETCH);
 //   1. theta, v and the M replica slices arrive in shared memory by bulk
 //      copies (cp.async.bulk, one per array, issued by thread 0 and
 //      completing on the CTA's mbarrier; every thread's wait on it is
@@ -19,26 +23,32 @@
 //      m turns worker m's maximum into its scale and reciprocal;
 //   3. the workers' pseudo-gradients are encoded, decoded and summed in FP32
 //      worker order, reading the replicas again from shared memory;
-//   4. the mean is encoded and decoded once (its block maximum is barrier 2).
+//   4. the mean (the sum over M: a product where M is a power of two) is
+//      encoded and decoded once on pairs (its block maximum is barrier 2).
 //      Every thread has then read this block's staging, so thread 0 issues
 //      the next block's bulk copies into the same buffer; they overlap the
 //      outer step and the stores;
-//   5. theta' is written once, in the replica type, to an output tile in
-//      shared memory (theta' and v' in fp32 too where they fit), and after
-//      the next block's barrier 1 thread 0 stores the tiles with bulk
-//      copies: the M replica resets are M copies of one tile.  Before
-//      barrier 2 of that block it waits until they have read the tiles.
-// Drift energies sum in fp32 per thread over at most 8 blocks (32 squares)
-// before each warp adds them, in a fixed order, to its fp64 row.  The
-// arithmetic of every element is the split form's (aloco_int8.cu), so both
-// forms give the same codes, scales and outputs.
+//   5. the outer step runs on pairs, 4 elements at a time, and theta' is
+//      written once, in the replica type, to an output tile in shared
+//      memory (theta' and v' in fp32 too where they fit); after the next
+//      block's barrier 1 thread 0 stores the tiles with bulk copies: the M
+//      replica resets are M copies of one tile.  Before barrier 2 of that
+//      block it waits until they have read the tiles.
+// Drift energies: for bf16 with more than 8 workers each block's energies
+// are summed across the warp at once (recursive halving) into fp64 rows;
+// elsewhere fp32 accumulators over up to 8 blocks (at most 64 squares a
+// thread) are reduced worker by worker, in a fixed order.  The squared
+// decoded means take the second route in every shape.  The arithmetic of
+// every element is the split form's (aloco_int8.cu): the paired operations
+// round each lane as the scalar ones do, so both forms give the same codes,
+// scales and outputs.
 //
 // Shared memory per CTA: the input buffer, 4096 x (8 + G x element size)
 // bytes for a group of G workers, and the output tiles, 4096 x element size
 // (plus 4096 x 8 for the fp32 theta' and v' tiles where they fit; elsewhere
 // threads store theta' and v' themselves).  One group holds every worker for
 // bf16 and for fp32 up to M = 8; fp32 with 9 <= M <= 16 stages each block's
-// replicas in groups of about three workers (see fused_group).
+// replicas in groups of at most five workers (see fused_group).
 //
 // A bounded wait that runs out (about 2 s) sets the round's error word; the
 // whole CTA leaves the block loop together at the next barrier, thread 0
@@ -53,6 +63,43 @@ namespace aloco {
 namespace {
 
 constexpr int kFlushBlocks = 8;
+
+// A hint to bring `bytes` (multiple of 16, 16-byte aligned address) of
+// global memory into L2 under the cache policy `pol` (createpolicy); nothing
+// waits for it and nothing is written.
+__device__ __forceinline__ void bulk_prefetch_l2_hint(const void *src, uint32_t bytes,
+                                                      uint64_t pol) {
+    asm volatile("cp.async.bulk.prefetch.L2.global.L2::cache_hint [%0], %1, %2;" ::"l"(src),
+                 "r"(bytes), "l"(pol)
+                 : "memory");
+}
+// A bulk load (as bulk_load) with an L2 cache policy
+__device__ __forceinline__ void bulk_load_hint(uint32_t dst, const void *src, uint32_t bytes,
+                                               uint32_t bar, uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint "
+        "[%0], [%1], %2, [%3], %4;" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar), "l"(pol)
+        : "memory");
+}
+// A bulk store (as bulk_store) with an L2 cache policy
+__device__ __forceinline__ void bulk_store_hint(void *dst, uint32_t src, uint32_t bytes,
+                                                uint64_t pol) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(dst),
+                 "r"(src), "r"(bytes), "l"(pol)
+                 : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
 constexpr int kFusedMax = 16;
 
 // Shared memory of one SM and the largest a CTA may take (bytes), and the
@@ -99,11 +146,17 @@ __host__ __device__ constexpr int fused_group() {
     if (grouped_direct<M, BF16>()) return balanced_group(M, ALOCO_I8_GDIRECT);
     return balanced_group(M, 3);
 }
-// the static shared arrays of the kernel and of the final reduction (an
-// upper bound)
-template <int M, int T>
+// The static shared arrays of the kernel and of the final reduction, per
+// warp: the group's warp maxima (4 G), the mean's (4), the energy rows
+// (8 (M + 1)), the scale table (8 (G + 1)), the reduction's rows (8 (M + 1))
+// and non-finite counts (8); plus 256 bytes for the mbarrier and scalars.
+// An upper bound of what ptxas reports for every instantiation.
+template <int M, bool BF16, int T>
 __host__ __device__ constexpr size_t static_bytes() {
-    return (size_t)(T / 32) * (4 * M + 4 + 8 * M + 8 * (M + 1)) + 4096;
+    return (size_t)(T / 32) *
+               (4 * fused_group<M, BF16>() + 4 + 8 * (M + 1) +
+                8 * (fused_group<M, BF16>() + (fused_group<M, BF16>() & 1)) + 8 * (M + 1) + 8) +
+           256;
 }
 // shared memory one of C CTAs per SM may take
 template <int C>
@@ -116,13 +169,13 @@ __host__ __device__ constexpr size_t cta_budget() {
 template <int M, bool BF16>
 __host__ __device__ constexpr bool fits_two_staged() {
     return (size_t)kI8Block * (8 + fused_group<M, BF16>() * esize<BF16>()) +
-               (size_t)kI8Block * esize<BF16>() + static_bytes<M, 512>() <=
+               (size_t)kI8Block * esize<BF16>() + static_bytes<M, BF16, 512>() <=
            cta_budget<2>();
 }
 template <int M, bool BF16>
 __host__ __device__ constexpr bool fits_two_direct() {
     return (size_t)kI8Block * (fused_group<M, BF16>() * esize<BF16>()) +
-               (size_t)kI8Block * esize<BF16>() + static_bytes<M, 512>() <=
+               (size_t)kI8Block * esize<BF16>() + static_bytes<M, BF16, 512>() <=
            cta_budget<2>();
 }
 // theta and v are not staged where that alone keeps two CTAs per SM from
@@ -158,7 +211,7 @@ __host__ __device__ constexpr size_t in_bytes() {
 template <int M, bool BF16, int T, int C>
 __host__ __device__ constexpr bool tile_gv() {
     return in_bytes<M, BF16>() + (size_t)kI8Block * (esize<BF16>() + (BF16 ? 8 : 4)) +
-               static_bytes<M, T>() <=
+               static_bytes<M, BF16, T>() <=
            cta_budget<C>();
 }
 template <int M, bool BF16, int T, int C>
@@ -172,8 +225,50 @@ __host__ __device__ constexpr size_t fused_smem() {
 }
 template <int M, bool BF16, int T, int C>
 __host__ __device__ constexpr bool fits() {
-    return fused_smem<M, BF16, T, C>() + static_bytes<M, T>() <= cta_budget<C>();
+    return fused_smem<M, BF16, T, C>() + static_bytes<M, BF16, T>() <= cta_budget<C>();
 }
+
+// Blocks ahead whose arrays thread 0 asks L2 to fetch (cp.async.bulk
+// .prefetch.L2) as each block starts, so that the bulk copy of the next block
+// into shared memory, issued at barrier 2, reads L2 instead of HBM.  With
+// one CTA per SM nothing else runs while that copy lands.  The prefetch
+// marks its lines evict-last, and the copies that read a block into shared
+// memory and the bulk stores mark theirs evict-first (each is used once), so
+// prefetched lines stay until their copy: DRAM reads 1.016x the algorithmic
+// bytes on 2^26 x 16 bf16, against 1.225x with no policies.  Measured on
+// GB300 (4e8 parameters, fraction of the copy peak), one block ahead against
+// none: bf16 M = 16 0.933 (0.846), M = 13 0.928 (0.818); M = 14 0.922, M = 15
+// 0.925; without the policies 0.894 and 0.895 (M = 16, 13), with only the
+// evict-last prefetch 0.902 and 0.899, with evict-first loads but plain
+// stores 0.920 and 0.916; evict-first loads and stores on every shape lost
+// 2-3 % on the shapes without prefetch.  The prefetch (before the policies)
+// lost on fp32 with one CTA per SM (M = 8 0.83 against 0.99, M = 6 0.91
+// against 0.95, the 150M set 0.83 against 0.95) and with two CTAs per SM
+// (bf16 M = 8 0.78 against 0.95, M = 12 0.72 against 0.86, fp32 M = 16 0.65
+// against 0.93); two blocks ahead lost everywhere.  -1 (default): one block
+// ahead where bf16 runs one CTA per SM, none elsewhere; otherwise the
+// number of blocks ahead everywhere (tuning knobs).
+#ifndef ALOCO_I8_PREFETCH
+#define ALOCO_I8_PREFETCH -1
+#endif
+
+// Where the next block is located: thread 0 locates it as a block starts
+// and leaves it in shared memory for every thread, so the next block's
+// copies go out at barrier 2 without a search before them; or thread 0
+// searches at barrier 2 and every thread at the end of the block.  On flat
+// vectors both cost a few instructions; which is faster depends on the code
+// ptxas makes of the rest.  Measured on GB300 over every shape (fraction of
+// the copy peak, shared memory against searching): the 150M set (fp32 M = 8,
+// one CTA per SM, 111 tensor parts) 0.954 (0.926); bf16 M = 9 0.959 (0.896),
+// M = 10 0.953 (0.886), M = 11 0.937 (0.862), M = 12 0.924 (0.918), M = 13..16
+// within 0.7 %; searching: bf16 M = 6 0.946 (0.899), fp32 M = 12 0.942
+// (0.884), M = 16 0.934 (0.898), M = 3 0.942 (0.930), the 3B set (bf16 M = 8)
+// 0.957 (0.947), the 1B set 0.982 (0.977); the other shapes within 0.5 %.
+// So shared memory where one CTA runs per SM and for bf16 with M > 8.
+// ALOCO_I8_NEXT_SMEM = 0 or 1 forces either everywhere (tuning knobs).
+#ifndef ALOCO_I8_NEXT_SMEM
+#define ALOCO_I8_NEXT_SMEM 2
+#endif
 
 // Threads per CTA (T) and elements per thread (4096 / T), measured on
 // GB300 (2^26-parameter rounds, fraction of the measured copy peak):
@@ -203,15 +298,53 @@ __host__ __device__ constexpr int fused_ctas() {
     if (ALOCO_I8_FUSED_CTAS) return ALOCO_I8_FUSED_CTAS;
     return (T == 512 && fits<M, BF16, 512, 2>()) ? 2 : 1;
 }
-
-// A thread's replica values of staging slots m0 and m0 + 1 (when m0 + 1 <
-// lim, the slots in use),
-// widened exactly, as PER / 2 pairs each.  Worker m's slice starts at
-// m x 4096 x element size; thread t's chunks of 4 elements sit at 4t + c x 4T.
+// bf16 on one CTA per SM (M >= 13): the shapes where the L2 prefetch and
+// the mixed-precision subtraction measured faster
 template <int M, bool BF16, int T>
+__host__ __device__ constexpr bool bf16_one_cta() {
+    return BF16 && fused_ctas<M, BF16, T>() == 1;
+}
+
+// bf16 replicas may enter theta - x through the mixed-precision FMA (bf16
+// operands, fp32 addend and result): fl(theta - x) in one instruction per
+// element from the staged word, with no separate widening; otherwise each
+// pair is widened and subtracted with the paired FMA.  Both round every
+// element the same way.  Measured on GB300 (4e8 parameters, fraction of the
+// copy peak) against widened pairs: bf16 M = 9 0.956 (0.942), M = 10 0.953
+// (0.920), M = 11 0.935 (0.900), M = 12 0.923 (0.881), M = 16 0.894 (0.863);
+// M = 8 0.865 (0.952).  ALOCO_I8_MIXED = 0 never takes it, 1 always (for
+// bf16), 2 (default) for bf16 with M > 8 (tuning knobs).
+#ifndef ALOCO_I8_MIXED
+#define ALOCO_I8_MIXED 2
+#endif
+// A pair of replica values as held between the staging and the
+// subtraction: a word of two bf16 values (RAW), or two fp32 values.
+template <bool RAW>
+using RepPair = typename std::conditional<RAW, uint32_t, float2>::type;
+
+// fl(theta - x) of a pair
+__device__ __forceinline__ float2 dpair(float2 g, float2 x) { return sub2(g, x); }
+__device__ __forceinline__ float2 dpair(float2 g, uint32_t w) {
+    // x (-1) + theta, one rounding per element: the rounding of sub2's lanes
+    float2 d;
+    asm("{\n\t.reg .b16 lo, hi, m1;\n\t"
+        "mov.b32 {lo, hi}, %2;\n\t"
+        "mov.b16 m1, 0xBF80;\n\t"
+        "fma.rn.f32.bf16 %0, lo, m1, %3;\n\t"
+        "fma.rn.f32.bf16 %1, hi, m1, %4;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "r"(w), "f"(g.x), "f"(g.y));
+    return d;
+}
+
+// A thread's replica pairs of staging slots m0 and m0 + 1 (when m0 + 1 <
+// lim, the slots in use), PER / 2 pairs each.  Worker m's slice starts at
+// m x 4096 x element size; thread t's chunks of 4 elements sit at 4t + c x 4T.
+template <int M, bool BF16, int T, bool RAW>
 __device__ __forceinline__ void staged_reps(const unsigned char *sx, int m0, int t,
-                                            float2 (&a)[kI8Block / T / 2],
-                                            float2 (&b)[kI8Block / T / 2], int lim = M) {
+                                            RepPair<RAW> (&a)[kI8Block / T / 2],
+                                            RepPair<RAW> (&b)[kI8Block / T / 2], int lim = M) {
+    static_assert(BF16 || !RAW, "raw words hold bf16 pairs");
     constexpr int PER = kI8Block / T;
     constexpr int ES = esize<BF16>();
     const unsigned char *p0 = sx + (size_t)m0 * kI8Block * ES + 4 * t * ES;
@@ -221,12 +354,20 @@ __device__ __forceinline__ void staged_reps(const unsigned char *sx, int m0, int
         const int off = c * 4 * T * ES;
         if constexpr (BF16) {
             const uint2 w = *reinterpret_cast<const uint2 *>(p0 + off);
-            a[2 * c] = make_float2(bf16_lo(w.x), bf16_hi(w.x));
-            a[2 * c + 1] = make_float2(bf16_lo(w.y), bf16_hi(w.y));
-            if (m0 + 1 < lim) {
-                const uint2 u = *reinterpret_cast<const uint2 *>(p1 + off);
-                b[2 * c] = make_float2(bf16_lo(u.x), bf16_hi(u.x));
-                b[2 * c + 1] = make_float2(bf16_lo(u.y), bf16_hi(u.y));
+            const uint2 u = m0 + 1 < lim ? *reinterpret_cast<const uint2 *>(p1 + off)
+                                         : make_uint2(0u, 0u);
+            if constexpr (RAW) {
+                a[2 * c] = w.x;
+                a[2 * c + 1] = w.y;
+                b[2 * c] = u.x;
+                b[2 * c + 1] = u.y;
+            } else {
+                a[2 * c] = make_float2(bf16_lo(w.x), bf16_hi(w.x));
+                a[2 * c + 1] = make_float2(bf16_lo(w.y), bf16_hi(w.y));
+                if (m0 + 1 < lim) {
+                    b[2 * c] = make_float2(bf16_lo(u.x), bf16_hi(u.x));
+                    b[2 * c + 1] = make_float2(bf16_lo(u.y), bf16_hi(u.y));
+                }
             }
         } else {
             const float4 q = *reinterpret_cast<const float4 *>(p0 + off);
@@ -264,13 +405,13 @@ __device__ __forceinline__ float block_amax(const float (&y)[PER], unsigned *red
 // 0.911 (4e8 parameters and the 3B set alike); bf16 M = 16 0.729 against
 // 0.741 (24 bytes of register spills appear at 64 registers); fp32 M = 12
 // unchanged.  So it is taken for bf16 with M <= 8.  ALOCO_I8_FAST = 0 turns
-// it off everywhere (a tuning knob).
+// it off everywhere, 2 takes it everywhere (a tuning knob).
 #ifndef ALOCO_I8_FAST
 #define ALOCO_I8_FAST 1
 #endif
 template <int M, bool BF16>
 __host__ __device__ constexpr bool i8_fast() {
-    return ALOCO_I8_FAST && BF16 && M <= 8;
+    return ALOCO_I8_FAST == 2 || (ALOCO_I8_FAST && BF16 && M <= 8);
 }
 
 // max(a, b, c), ignoring NaN operands (as fmaxf)
@@ -297,6 +438,133 @@ __device__ __forceinline__ float2 code2_fast_max(float2 y, float r, float &far) 
     return n;
 }
 
+// Block-wide max |y| of a thread's pairs, as float bits: each warp's
+// maximum goes to red[warp]; after the barrier every warp folds the W values
+// with one warp max.  A NaN wins (the NaN-propagating maximum gives the
+// canonical NaN, whose bits exceed +inf's), as in block_amax.
+template <int NP, int W>
+__device__ __forceinline__ float block_amax2(const float2 (&y)[NP], unsigned *red) {
+    float mf = 0.f;
+#pragma unroll
+    for (int j = 0; j < NP; ++j) mf = max3_nan(mf, fabsf(y[j].x), fabsf(y[j].y));
+    const unsigned m = __reduce_max_sync(0xffffffffu, __float_as_uint(mf));
+    const int lane = threadIdx.x & 31;
+    if (lane == 0) red[threadIdx.x >> 5] = m;
+    __syncthreads();
+    return __uint_as_float(__reduce_max_sync(0xffffffffu, lane < W ? red[lane] : 0u));
+}
+
+// fl32(sum / M) of every pair, the quotient div_by_scale gives.  For M a
+// power of two the quotient is the product with 1/M (exact): both round the
+// same real number, so they agree, underflow included.  Otherwise the
+// Markstein steps of div_by_scale run on pairs, and a thread with a
+// non-finite quotient redoes its elements with div_by_scale itself.
+template <int M, int NP>
+__device__ __forceinline__ void mean_of_sum(const float2 (&sum)[NP], float2 (&mean)[NP]) {
+    if constexpr ((M & (M - 1)) == 0) {
+#pragma unroll
+        for (int j = 0; j < NP; ++j) mean[j] = mul2_rn(sum[j], splat2(1.f / (float)M));
+    } else {
+        const float fM = (float)M, rM = __frcp_rn(fM);
+        float bad = 0.f;
+#pragma unroll
+        for (int j = 0; j < NP; ++j) {
+            const float2 q0 = mul2_rn(sum[j], splat2(rM));
+            const float2 q1 =
+                __ffma2_rn(__ffma2_rn(splat2(-fM), q0, sum[j]), splat2(rM), q0);
+            mean[j] = __ffma2_rn(__ffma2_rn(splat2(-fM), q1, sum[j]), splat2(rM), q1);
+            bad = max3_nan(bad, fabsf(mean[j].x), fabsf(mean[j].y));
+        }
+        if (!(bad <= FLT_MAX)) {
+#pragma unroll
+            for (int j = 0; j < NP; ++j)
+                mean[j] = make_float2(div_by_scale(sum[j].x, fM, rM),
+                                      div_by_scale(sum[j].y, fM, rM));
+        }
+    }
+}
+
+// Decoded codes fl32(code(y) s) of a thread's pairs under the block's own
+// scale s (r = fl32(1/s)): the product path of code2_fast_max, and a warp
+// whose products are not all provably the quotient's takes every element
+// through codec_code_f (codec_code_fast's slow path); the other lanes'
+// codes do not change.  Every finite product is below 127.5 here (see
+// code2_fast), so no clipping is needed on the product path.
+template <int NP>
+__device__ __forceinline__ void decode_mean(const float2 (&y)[NP], float s, float r,
+                                            float2 (&dq)[NP]) {
+    float2 n[NP];
+    float far = 0.f;
+#pragma unroll
+    for (int j = 0; j < NP; ++j) n[j] = code2_fast_max(y[j], r, far);
+    if (__any_sync(0xffffffffu, !(far < kCodeMargin))) {
+#pragma unroll
+        for (int j = 0; j < NP; ++j)
+            n[j] = make_float2(codec_code_f(y[j].x, s, r), codec_code_f(y[j].y, s, r));
+    }
+#pragma unroll
+    for (int j = 0; j < NP; ++j) dq[j] = mul2_rn(n[j], splat2(s));
+}
+
+// outer_step on a pair: the same operations, each lane rounded as the
+// scalar step rounds it.
+__device__ __forceinline__ void outer_step2(const Coef &k, float2 s, float2 g, float2 v,
+                                            float2 &gp, float2 &vp) {
+    const float2 dt = __ffma2_rn(s, splat2(k.c_hi), __fmul2_rn(s, splat2(k.c_lo)));
+    vp = __ffma2_rn(splat2(k.mu_hi), v, __ffma2_rn(splat2(k.mu_lo), v, dt));
+    const float2 d = __ffma2_rn(splat2(k.mu_hi), vp, __ffma2_rn(splat2(k.mu_lo), vp, dt));
+    gp = add2_rn(g, __ffma2_rn(splat2(k.ne_hi), d, __fmul2_rn(splat2(k.ne_lo), d)));
+}
+
+// Warp sums of the P values each lane holds (P a power of two, at most 32)
+// by recursive halving: at each step a lane keeps the half of its values
+// that its lane bit selects and adds the partner's copy of that half; the
+// last steps add across the lanes that share a value.  Lane L returns the
+// warp sum of value L >> (5 - log2 P).  The order is fixed (and a + b = b + a
+// exactly), so every lane holding a value has the same bits.
+template <int P>
+__device__ __forceinline__ float warp_sum_scatter(float (&v)[P]) {
+    static_assert(P >= 1 && P <= 32 && (P & (P - 1)) == 0, "P: a power of two");
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int st = 0; st < 5; ++st) {
+        const int mask = 16 >> st;
+        const int n = P >> st;  // values still held
+        if (n > 1) {
+            const bool up = (lane & mask) != 0;
+#pragma unroll
+            for (int i = 0; i < n / 2; ++i) {
+                const float send = up ? v[i] : v[i + n / 2];
+                const float keep = up ? v[i + n / 2] : v[i];
+                v[i] = keep + __shfl_xor_sync(0xffffffffu, send, mask);
+            }
+        } else {
+            v[0] += __shfl_xor_sync(0xffffffffu, v[0], mask);
+        }
+    }
+    return v[0];
+}
+__host__ __device__ constexpr int pow2_at_least(int n) {
+    return n <= 1 ? 1 : 2 * pow2_at_least((n + 1) / 2);
+}
+
+// The workers' energies of a block summed across the warp at once (warp
+// sums by recursive halving, one fp64 row update per worker and block), so
+// no per-worker accumulator stays live through the rest of the block.
+// Measured on GB300 (4e8 parameters, fraction of the copy peak) against fp32
+// accumulators over up to 8 blocks reduced worker by worker: bf16 M = 16
+// 0.832 (0.744), M = 12 0.888 (0.861), M = 8 0.947 (0.953); fp32 M = 16
+// (groups, whose energies are reduced per group and block anyway) 0.931
+// (0.932).  Taken for bf16 with M > 8.  ALOCO_I8_EROW = 0 turns it off, 1
+// takes it for every single-group shape (tuning knobs).
+#ifndef ALOCO_I8_EROW
+#define ALOCO_I8_EROW 2
+#endif
+template <int M, bool BF16>
+__host__ __device__ constexpr bool erow() {
+    return ALOCO_I8_EROW == 1 || (ALOCO_I8_EROW == 2 && BF16 && M > 8);
+}
+
 }  // namespace
 
 template <int M, bool BF16, int T>
@@ -307,12 +575,23 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     constexpr int NP = PER / 2;        // pairs per thread
     constexpr int W = T / 32;          // warps
     constexpr int ES = esize<BF16>();
+    // blocks between the warp reductions of the fp32 accumulators: at most
+    // 64 squares a thread
+    constexpr int kFlush = kFlushBlocks;
     constexpr bool GV = tile_gv<M, BF16, T, fused_ctas<M, BF16, T>()>();
     constexpr int G = fused_group<M, BF16>();    // workers staged at a time
     constexpr int NG = (M + G - 1) / G;          // groups per block
     constexpr bool GROUPED = NG > 1;
     constexpr int EA = GROUPED ? G : M;          // energy accumulators a thread
     constexpr bool DGV = direct_gv<M, BF16>();   // theta, v read from global memory
+    constexpr bool EROW = !GROUPED && erow<M, BF16>();  // energies reduced every block
+    constexpr int PF = ALOCO_I8_PREFETCH >= 0 ? ALOCO_I8_PREFETCH
+                                              : (bf16_one_cta<M, BF16, T>() ? 1 : 0);
+    constexpr bool NEXT_SMEM =
+        ALOCO_I8_NEXT_SMEM == 1 ||
+        (ALOCO_I8_NEXT_SMEM == 2 && (fused_ctas<M, BF16, T>() == 1 || (BF16 && M > 8)));
+    // bf16 pairs reach the subtraction as raw words (see ALOCO_I8_MIXED)
+    constexpr bool MIX = BF16 && (ALOCO_I8_MIXED == 1 || (ALOCO_I8_MIXED == 2 && M > 8));
     constexpr uint32_t kGVBytes = kI8Block * 4;  // one fp32 array of a block
     constexpr uint32_t kXBytes = kI8Block * ES;  // one replica slice
     // Single buffers suffice: red_w is read between a group's first barrier
@@ -320,7 +599,14 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     // barrier 2 and rewritten only after the next block's first barrier.
     __shared__ unsigned red_w[G][W];                  // [worker][warp]: conflict-free reads
     __shared__ unsigned red1[W];
-    __shared__ double e_w[W][M];
+    __shared__ double e_w[W][M + 1];   // [warp][worker energies, then sum Dbar^2]
+    __shared__ int64_t s_pstart;        // thread 0: start of the block whose tiles wait
+    // the next block's start and length, located by thread 0 as a block
+    // starts and read by every thread after barrier 1 (two slots by the
+    // parity of the iteration: a slot is rewritten only after every thread
+    // has passed the next barrier 1)
+    __shared__ int64_t s_nstart[2];
+    __shared__ int s_nlen[2];
     __shared__ __align__(16) float2 sr[W][G + (G & 1)];  // per warp: (scale, 1/scale)
     __shared__ __align__(8) unsigned long long full_bar;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -334,7 +620,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     const uint32_t bar = smem_addr(&full_bar);
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    if (lane < M) e_w[warp][lane] = 0.0;
+    if (lane <= M) e_w[warp][lane] = 0.0;
     if (t == 0) {
         mbar_init(bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -357,16 +643,31 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
             e_acc[m] = 0.f;
         }
     };
+    float b32 = 0.f;  // sum of squared decoded means since the last flush
+    auto flush_b = [&]() {
+        float e = b32;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) e += __shfl_down_sync(0xffffffffu, e, off);
+        if (lane == 0) e_w[warp][M] += (double)e;
+        b32 = 0.f;
+    };
+    // energies of one block, all M workers: warp sums by recursive halving
+    // into the fp64 rows
+    constexpr int EP = pow2_at_least(M);
+    auto add_rows = [&](float (&eb)[EP]) {
+        const float e = warp_sum_scatter<EP>(eb);
+        const int w = lane >> (5 - __builtin_ctz(EP));  // the row this lane holds
+        if ((lane & (32 / EP - 1)) == 0 && w < M) e_w[warp][w] += (double)e;
+    };
     auto flush = [&]() {
-        flush_rows(0, EA);
+        if constexpr (!GROUPED && !EROW) flush_rows(0, EA);
+        flush_b();
         since_flush = 0;
     };
 
-    float b32 = 0.f;
-    double b64 = 0.0;
     unsigned nf = 0;
     const Coef k{a.c_hi, a.c_lo, a.mu_hi, a.mu_lo, a.neg_eta_hi, a.neg_eta_lo};
-    const int64_t nblocks = P.blk[P.n_parts];
+    const int nblocks = (int)P.blk[P.n_parts];  // below 2^31 - grid (host check)
     // thread t holds the 4-element chunks at 4t + c x 4T (c < PER / 4), so
     // every warp access to a staged array is contiguous
     auto el = [&](int i) { return (i >> 2) * (4 * T) + 4 * t + (i & 3); };
@@ -399,17 +700,48 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         const int m0 = q * G;
         const int gq = M - m0 < G ? M - m0 : G;
         mbar_arrive_expect_tx(bar, (q == 0 && !DGV ? 2 * kGVBytes : 0) + gq * kXBytes);
-        if (q == 0 && !DGV) {
-            bulk_load(smem_addr(sg), a.g + s, kGVBytes, bar);
-            bulk_load(smem_addr(sv), a.v + s, kGVBytes, bar);
-        }
+        if constexpr (PF > 0) {
+            // read once: evict these lines first, ahead of the prefetched ones
+            const uint64_t pol = policy_evict_first();
+            if (q == 0 && !DGV) {
+                bulk_load_hint(smem_addr(sg), a.g + s, kGVBytes, bar, pol);
+                bulk_load_hint(smem_addr(sv), a.v + s, kGVBytes, bar, pol);
+            }
 #pragma unroll
-        for (int m = 0; m < G; ++m)
-            if (m < gq)
-                bulk_load(smem_addr(sx + m * kXBytes),
-                          reinterpret_cast<const unsigned char *>(a.x[m0 + m]) + s * ES,
-                          kXBytes, bar);
+            for (int m = 0; m < G; ++m)
+                if (m < gq)
+                    bulk_load_hint(smem_addr(sx + m * kXBytes),
+                                   reinterpret_cast<const unsigned char *>(a.x[m0 + m]) + s * ES,
+                                   kXBytes, bar, pol);
+        } else {
+            if (q == 0 && !DGV) {
+                bulk_load(smem_addr(sg), a.g + s, kGVBytes, bar);
+                bulk_load(smem_addr(sv), a.v + s, kGVBytes, bar);
+            }
+#pragma unroll
+            for (int m = 0; m < G; ++m)
+                if (m < gq)
+                    bulk_load(smem_addr(sx + m * kXBytes),
+                              reinterpret_cast<const unsigned char *>(a.x[m0 + m]) + s * ES,
+                              kXBytes, bar);
+        }
         in_flight = true;
+    };
+    // thread 0: the L2 prefetch of every array of the block kbi (whole,
+    // aligned blocks only)
+    auto prefetch_block = [&](int64_t kbi) {
+        if (kbi >= nblocks) return;
+        int64_t ps;
+        int pl;
+        locate_block(P, kbi, ps, pl);
+        if (!bulk_block(ps, pl)) return;
+        const uint64_t pol = policy_evict_last();
+        bulk_prefetch_l2_hint(a.g + ps, kGVBytes, pol);
+        bulk_prefetch_l2_hint(a.v + ps, kGVBytes, pol);
+#pragma unroll
+        for (int m = 0; m < M; ++m)
+            bulk_prefetch_l2_hint(reinterpret_cast<const unsigned char *>(a.x[m]) + ps * ES,
+                                  kXBytes, pol);
     };
     // every thread: its own elements of group q of a short or unaligned block
     auto stage_own = [&](int64_t s, int l, int q) {
@@ -440,23 +772,35 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
     };
     // thread 0: the output tiles of the block at s go to global memory
     auto store_tiles = [&](int64_t s) {
-        if constexpr (GV) {
-            bulk_store(a.g + s, smem_addr(og), kGVBytes);
-            bulk_store(a.v + s, smem_addr(ov), kGVBytes);
-        }
+        if constexpr (PF > 0) {
+            // written once: evict these lines first, ahead of the prefetched ones
+            const uint64_t pol = policy_evict_first();
+            if constexpr (GV) {
+                bulk_store_hint(a.g + s, smem_addr(og), kGVBytes, pol);
+                bulk_store_hint(a.v + s, smem_addr(ov), kGVBytes, pol);
+            }
 #pragma unroll
-        for (int m = 0; m < M; ++m)
-            bulk_store(reinterpret_cast<unsigned char *>(a.x[m]) + s * ES, smem_addr(ox),
-                       kXBytes);
+            for (int m = 0; m < M; ++m)
+                bulk_store_hint(reinterpret_cast<unsigned char *>(a.x[m]) + s * ES, smem_addr(ox),
+                                kXBytes, pol);
+        } else {
+            if constexpr (GV) {
+                bulk_store(a.g + s, smem_addr(og), kGVBytes);
+                bulk_store(a.v + s, smem_addr(ov), kGVBytes);
+            }
+#pragma unroll
+            for (int m = 0; m < M; ++m)
+                bulk_store(reinterpret_cast<unsigned char *>(a.x[m]) + s * ES, smem_addr(ox),
+                           kXBytes);
+        }
         bulk_commit();
     };
 
-    int64_t kb = blockIdx.x;
+    int kb = blockIdx.x;
     int64_t start = 0;
     int len = 0;
     uint32_t phase = 0;
     bool pend = false;  // the previous block's tiles wait for their bulk stores
-    int64_t pstart = 0;
     bool failed = false;
     if (kb < nblocks) {
         locate_block(P, kb, start, len);
@@ -465,14 +809,19 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         else if (t == 0)
             stage_bulk(kb, start, 0);
     }
-    for (; kb < nblocks; kb += gridDim.x) {
+    int par = 0;
+    for (; kb < nblocks; kb += gridDim.x, par ^= 1) {
+        if (PF > 0 && t == 0) prefetch_block(kb + PF * (int64_t)gridDim.x);
         const bool full = len == kI8Block;
         const bool bulk = bulk_block(start, len);
-        const int64_t nk = kb + gridDim.x;
-        int64_t nstart = 0;
-        int nlen = 0;
-        if (nk < nblocks) locate_block(P, nk, nstart, nlen);
-        const bool next_bulk = nk < nblocks && bulk_block(nstart, nlen);
+        const int nk = kb + gridDim.x;  // the next block
+        if (NEXT_SMEM && t == 0 && nk < nblocks) {
+            int64_t ns;
+            int nl;
+            locate_block(P, nk, ns, nl);
+            s_nstart[par] = ns;
+            s_nlen[par] = nl;
+        }
         float g[PER];
         float2 g2[NP];    // theta, as pairs
         float2 sum2[NP];  // the workers' decoded sum
@@ -500,10 +849,13 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
             for (int j = 0; j < NP; ++j) g2[j] = make_float2(g[2 * j], g[2 * j + 1]);
 
             // 2. block maxima and energies of every worker
-            auto worker_max = [&](int m, const float2 (&x)[NP]) {
+            float eb[EP];  // this block's energies (EROW)
+#pragma unroll
+            for (int m = 0; m < EP; ++m) eb[m] = 0.f;
+            auto worker_max = [&](int m, const RepPair<MIX> (&x)[NP]) {
                 float2 d[NP];
 #pragma unroll
-                for (int j = 0; j < NP; ++j) d[j] = sub2(g2[j], x[j]);
+                for (int j = 0; j < NP; ++j) d[j] = dpair(g2[j], x[j]);
                 float mf = 0.f;
                 float2 e2 = __fmul2_rn(d[0], d[0]);
 #pragma unroll
@@ -523,18 +875,19 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
                         mx = max(mx, max(__float_as_uint(fabsf(d[j].x)),
                                          __float_as_uint(fabsf(d[j].y))));
                 }
-                e_acc[m] += e;
+                if constexpr (EROW) eb[m] = e; else e_acc[m] += e;
                 mx = __reduce_max_sync(0xffffffffu, mx);
                 if (lane == 0) red_w[m][warp] = mx;
             };
 #pragma unroll
             for (int m = 0; m < M; m += 2) {
-                float2 xa[NP], xb[NP];
-                staged_reps<M, BF16, T>(sx, m, t, xa, xb);
+                RepPair<MIX> xa[NP], xb[NP];
+                staged_reps<M, BF16, T, MIX>(sx, m, t, xa, xb);
                 worker_max(m, xa);
                 if (m + 1 < M) worker_max(m + 1, xb);
             }
-            if (++since_flush == kFlushBlocks) flush();
+            if constexpr (EROW) add_rows(eb);
+            if (++since_flush == kFlush) flush();
             // barrier 1; a wait that ran out in any thread stops the whole CTA
             if (__syncthreads_or(timed_out)) {
                 failed = true;
@@ -542,7 +895,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
             }
             // every thread wrote its part of the previous block's tiles before
             // the barrier
-            if (pend && t == 0) store_tiles(pstart);
+            if (pend && t == 0) store_tiles(s_pstart);
             pend = false;
             {
                 // every warp folds the W warp maxima of each worker (lane w reads
@@ -565,25 +918,25 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
             // 3. encode, decode and sum in worker order
 #pragma unroll
             for (int j = 0; j < NP; ++j) sum2[j] = splat2(-0.f);
-            auto add_worker = [&](float2 scr, const float2 (&x)[NP]) {
+            auto add_worker = [&](float2 scr, const RepPair<MIX> (&x)[NP]) {
                 const float s = scr.x, r = scr.y;
                 bool ok = true;
                 float2 n[NP];
                 if constexpr (i8_fast<M, BF16>()) {
                     float far = 0.f;
 #pragma unroll
-                    for (int j = 0; j < NP; ++j) n[j] = code2_fast_max(sub2(g2[j], x[j]), r, far);
+                    for (int j = 0; j < NP; ++j) n[j] = code2_fast_max(dpair(g2[j], x[j]), r, far);
                     // warp-uniform: a lane that needs the exact quotient takes
                     // the whole warp through it (the same codes for the rest)
                     ok = !__any_sync(0xffffffffu, !(far < kCodeMargin));
                 } else {
 #pragma unroll
-                    for (int j = 0; j < NP; ++j) n[j] = code2_fast(sub2(g2[j], x[j]), r, ok);
+                    for (int j = 0; j < NP; ++j) n[j] = code2_fast(dpair(g2[j], x[j]), r, ok);
                 }
                 if (!ok) {
 #pragma unroll
                     for (int j = 0; j < NP; ++j) {
-                        const float2 d = sub2(g2[j], x[j]);
+                        const float2 d = dpair(g2[j], x[j]);
                         n[j] = make_float2(codec_code_f(d.x, s, r), codec_code_f(d.y, s, r));
                     }
                 }
@@ -597,8 +950,8 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
 #pragma unroll
             for (int m = 0; m < M; m += 2) {
                 const float4 scr = *reinterpret_cast<const float4 *>(&sr[warp][m]);
-                float2 xa[NP], xb[NP];
-                staged_reps<M, BF16, T>(sx, m, t, xa, xb);
+                RepPair<MIX> xa[NP], xb[NP];
+                staged_reps<M, BF16, T, MIX>(sx, m, t, xa, xb);
                 add_worker(make_float2(scr.x, scr.y), xa);
                 if (m + 1 < M) add_worker(make_float2(scr.z, scr.w), xb);
             }
@@ -631,10 +984,10 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
 
                 // 2. block maxima and energies of the group's workers (slot m of
                 // the staging holds worker m0 + m)
-                auto worker_max = [&](int m, const float2 (&x)[NP]) {
+                auto worker_max = [&](int m, const RepPair<MIX> (&x)[NP]) {
                     float2 d[NP];
 #pragma unroll
-                    for (int j = 0; j < NP; ++j) d[j] = sub2(g2[j], x[j]);
+                    for (int j = 0; j < NP; ++j) d[j] = dpair(g2[j], x[j]);
                     float mf = 0.f;
                     float2 e2 = __fmul2_rn(d[0], d[0]);
 #pragma unroll
@@ -661,15 +1014,17 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
 #pragma unroll
                 for (int m = 0; m < G; m += 2) {
                     if (m >= GQ) break;
-                    float2 xa[NP], xb[NP];
-                    staged_reps<G, BF16, T>(sx, m, t, xa, xb, GQ);
+                    RepPair<MIX> xa[NP], xb[NP];
+                    staged_reps<G, BF16, T, MIX>(sx, m, t, xa, xb, GQ);
                     worker_max(m, xa);
                     if (m + 1 < GQ) worker_max(m + 1, xb);
                 }
-                if constexpr (GROUPED)
+                if constexpr (GROUPED) {
                     flush_rows(m0, GQ);
-                else if (++since_flush == kFlushBlocks)
+                    if (q == 0 && ++since_flush == kFlush) flush();
+                } else if (++since_flush == kFlush) {
                     flush();
+                }
                 // barrier 1 (of the group); a wait that ran out in any thread
                 // stops the whole CTA
                 if (__syncthreads_or(timed_out)) {
@@ -679,7 +1034,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
                 if (q == 0) {
                     // every thread wrote its part of the previous block's tiles
                     // before the barrier
-                    if (pend && t == 0) store_tiles(pstart);
+                    if (pend && t == 0) store_tiles(s_pstart);
                     pend = false;
                 }
                 {
@@ -706,7 +1061,7 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
 #pragma unroll
                     for (int j = 0; j < NP; ++j) sum2[j] = splat2(-0.f);
                 }
-                auto add_worker = [&](float2 scr, const float2 (&x)[NP]) {
+                auto add_worker = [&](float2 scr, const RepPair<MIX> (&x)[NP]) {
                     const float sc = scr.x, r = scr.y;
                     bool ok = true;
                     float2 n[NP];
@@ -714,16 +1069,16 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
                         float far = 0.f;
 #pragma unroll
                         for (int j = 0; j < NP; ++j)
-                            n[j] = code2_fast_max(sub2(g2[j], x[j]), r, far);
+                            n[j] = code2_fast_max(dpair(g2[j], x[j]), r, far);
                         ok = !__any_sync(0xffffffffu, !(far < kCodeMargin));
                     } else {
 #pragma unroll
-                        for (int j = 0; j < NP; ++j) n[j] = code2_fast(sub2(g2[j], x[j]), r, ok);
+                        for (int j = 0; j < NP; ++j) n[j] = code2_fast(dpair(g2[j], x[j]), r, ok);
                     }
                     if (!ok) {
 #pragma unroll
                         for (int j = 0; j < NP; ++j) {
-                            const float2 d = sub2(g2[j], x[j]);
+                            const float2 d = dpair(g2[j], x[j]);
                             n[j] = make_float2(codec_code_f(d.x, sc, r), codec_code_f(d.y, sc, r));
                         }
                     }
@@ -738,8 +1093,8 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
                 for (int m = 0; m < G; m += 2) {
                     if (m >= GQ) break;
                     const float4 scr = *reinterpret_cast<const float4 *>(&sr[warp][m]);
-                    float2 xa[NP], xb[NP];
-                    staged_reps<G, BF16, T>(sx, m, t, xa, xb, GQ);
+                    RepPair<MIX> xa[NP], xb[NP];
+                    staged_reps<G, BF16, T, MIX>(sx, m, t, xa, xb, GQ);
                     add_worker(make_float2(scr.x, scr.y), xa);
                     if (m + 1 < GQ) add_worker(make_float2(scr.z, scr.w), xb);
                 }
@@ -761,93 +1116,124 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
 
         }
         // 4. the mean's codec
-        float v[PER];
+        float2 v2[NP];
         if constexpr (DGV) {
+            float v[PER];
             load_direct(v, a.v, start, len, bulk);
+#pragma unroll
+            for (int j = 0; j < NP; ++j) v2[j] = make_float2(v[2 * j], v[2 * j + 1]);
         } else {
 #pragma unroll
             for (int c = 0; c < PER; c += 4) {
                 const float4 q = *reinterpret_cast<const float4 *>(sv + el(c));
-                v[c] = q.x; v[c + 1] = q.y; v[c + 2] = q.z; v[c + 3] = q.w;
+                v2[c / 2] = make_float2(q.x, q.y);
+                v2[c / 2 + 1] = make_float2(q.z, q.w);
             }
         }
-        float sum[PER];
-#pragma unroll
-        for (int j = 0; j < NP; ++j) {
-            sum[2 * j] = sum2[j].x;
-            sum[2 * j + 1] = sum2[j].y;
-        }
-        const float fM = (float)M, rM = __frcp_rn(fM);
-#pragma unroll
-        for (int i = 0; i < PER; ++i) sum[i] = div_by_scale(sum[i], fM, rM);
+        float2 mean2[NP];
+        mean_of_sum<M, NP>(sum2, mean2);
         // the previous block's bulk stores have read the tiles before any
         // thread passes barrier 2 and rewrites them
         if (t == 0) bulk_wait_read();
         // barrier 2; elements beyond a short block hold 0 and do not move
         // the maximum
-        const float s = codec_scale(block_amax<PER, W>(sum, red1));
+        const float s = codec_scale(block_amax2<NP, W>(mean2, red1));
         // every thread has read this block's staging: the next block's bulk
         // copies go into the same buffer while the rest of this block runs
         // (a short or unaligned next block is staged after the stores)
-        if (next_bulk && t == 0) stage_bulk(nk, nstart, 0);
-        const float rs = __frcp_rn(s);
-        float gp[PER], vp[PER];
-#pragma unroll
-        for (int i = 0; i < PER; ++i) {
-            const float dq = __fmul_rn(codec_code_fast(sum[i], s, rs), s);
-            const bool in = full || el(i) < len;
-            if (in) b32 = fmaf(dq, dq, b32);
-            outer_step(k, dq, g[i], v[i], gp[i], vp[i]);
-            if (in) nf += not_finite(gp[i], vp[i]);
+        if constexpr (NEXT_SMEM) {
+            if (t == 0 && nk < nblocks && bulk_block(s_nstart[par], s_nlen[par]))
+                stage_bulk(nk, s_nstart[par], 0);
+        } else if (t == 0 && nk < nblocks) {
+            int64_t ns;
+            int nl;
+            locate_block(P, nk, ns, nl);
+            if (bulk_block(ns, nl)) stage_bulk(nk, ns, 0);
         }
-
-        // 5. the stores
-        if (bulk) {
+        // decode, outer step and stores chunk by chunk (4 elements), so a
+        // chunk's results alone are live
+        const float rs = __frcp_rn(s);
+        auto lo_hi = [](const float2 (&p)[2], int i) { return (i & 1) ? p[i >> 1].y : p[i >> 1].x; };
+        float2 b2 = splat2(0.f);
 #pragma unroll
-            for (int c = 0; c < PER; c += 4) {
+        for (int c = 0; c < PER; c += 4) {
+            const int j = c / 2;  // the chunk's first pair
+            const float2 y[2] = {mean2[j], mean2[j + 1]};
+            float2 dq[2], gp[2], vp[2];
+            decode_mean<2>(y, s, rs, dq);
+            // non-finite outputs are counted one by one only in a chunk
+            // that has one
+            float big = 0.f;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                if (full) b2 = __ffma2_rn(dq[h], dq[h], b2);
+                outer_step2(k, dq[h], g2[j + h], v2[j + h], gp[h], vp[h]);
+                big = max3_nan(big, fabsf(gp[h].x), fabsf(gp[h].y));
+                big = max3_nan(big, fabsf(vp[h].x), fabsf(vp[h].y));
+            }
+            if (!full) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    if (el(c + i) < len) b32 = fmaf(lo_hi(dq, i), lo_hi(dq, i), b32);
+            }
+            if (!(big <= FLT_MAX)) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    if (full || el(c + i) < len) nf += not_finite(lo_hi(gp, i), lo_hi(vp, i));
+            }
+
+            // 5. the stores
+            if (bulk) {
                 if constexpr (BF16) {
                     *reinterpret_cast<uint2 *>(ox + el(c) * 2) =
-                        make_uint2(pack_bf16x2(gp[c], gp[c + 1]), pack_bf16x2(gp[c + 2], gp[c + 3]));
+                        make_uint2(pack_bf16x2(gp[0].x, gp[0].y), pack_bf16x2(gp[1].x, gp[1].y));
                 }
                 if constexpr (GV || !BF16)
                     *reinterpret_cast<float4 *>(og + el(c)) =
-                        make_float4(gp[c], gp[c + 1], gp[c + 2], gp[c + 3]);
+                        make_float4(gp[0].x, gp[0].y, gp[1].x, gp[1].y);
                 if constexpr (GV)
                     *reinterpret_cast<float4 *>(ov + el(c)) =
-                        make_float4(vp[c], vp[c + 1], vp[c + 2], vp[c + 3]);
+                        make_float4(vp[0].x, vp[0].y, vp[1].x, vp[1].y);
                 if constexpr (!GV) {
                     __stcs(reinterpret_cast<float4 *>(a.g + start + el(c)),
-                           make_float4(gp[c], gp[c + 1], gp[c + 2], gp[c + 3]));
+                           make_float4(gp[0].x, gp[0].y, gp[1].x, gp[1].y));
                     __stcs(reinterpret_cast<float4 *>(a.v + start + el(c)),
-                           make_float4(vp[c], vp[c + 1], vp[c + 2], vp[c + 3]));
+                           make_float4(vp[0].x, vp[0].y, vp[1].x, vp[1].y));
                 }
-            }
-            fence_proxy_async_smem();  // the tiles are read by bulk copies
-            pend = true;
-            pstart = start;
-        } else {
+            } else {
 #pragma unroll
-            for (int i = 0; i < PER; ++i) {
-                const int e = el(i);
-                if (e >= len) continue;
-                a.g[start + e] = gp[i];
-                a.v[start + e] = vp[i];
+                for (int i = 0; i < 4; ++i) {
+                    const int e = el(c + i);
+                    if (e >= len) continue;
+                    const float gpi = lo_hi(gp, i);
+                    a.g[start + e] = gpi;
+                    a.v[start + e] = lo_hi(vp, i);
 #pragma unroll
-                for (int m = 0; m < M; ++m) {
-                    if constexpr (BF16)
-                        reinterpret_cast<__nv_bfloat16 *>(a.x[m])[start + e] =
-                            __float2bfloat16_rn(gp[i]);
-                    else
-                        reinterpret_cast<float *>(a.x[m])[start + e] = gp[i];
+                    for (int m = 0; m < M; ++m) {
+                        if constexpr (BF16)
+                            reinterpret_cast<__nv_bfloat16 *>(a.x[m])[start + e] =
+                                __float2bfloat16_rn(gpi);
+                        else
+                            reinterpret_cast<float *>(a.x[m])[start + e] = gpi;
+                    }
                 }
             }
         }
-        b64 += (double)b32;  // at most PER terms per thread and block
-        b32 = 0.f;
-        if (nk < nblocks && !next_bulk) stage_own(nstart, nlen, 0);
-
-        start = nstart;
-        len = nlen;
+        if (full) b32 += __fadd_rn(b2.x, b2.y);
+        if (bulk) {
+            fence_proxy_async_smem();  // the tiles are read by bulk copies
+            pend = true;
+            if (t == 0) s_pstart = start;
+        }
+        if (nk < nblocks) {
+            if constexpr (NEXT_SMEM) {
+                start = s_nstart[par];
+                len = s_nlen[par];
+            } else {
+                locate_block(P, nk, start, len);
+            }
+            if (!bulk_block(start, len)) stage_own(start, len, 0);
+        }
     }
     if (failed) {
         if (t == 0) {
@@ -857,12 +1243,22 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         }
     } else if (pend) {
         __syncthreads();
-        if (t == 0) store_tiles(pstart);
+        if (t == 0) store_tiles(s_pstart);
     }
     if (t == 0) bulk_wait_all();
-    if (since_flush > 0) flush();
+    // the energies still in registers, and the squared means of every block
+    // since the last flush (the last block's come after its flush check)
+    if constexpr (!GROUPED && !EROW) {
+        if (since_flush > 0) flush_rows(0, EA);
+    }
+    flush_b();
     __syncthreads();
     double e64[M];
+    double b64 = 0.0;
+    if (t == 0) {
+#pragma unroll
+        for (int w = 0; w < W; ++w) b64 += e_w[w][M];
+    }
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         double e = 0.0;
@@ -903,6 +1299,8 @@ cudaError_t fused_launch(const SyncArgs &a, const Int8Parts &P, int sm_count,
     if (grid > nblocks) grid = nblocks;
     if (grid > max_grid) grid = max_grid;
     if (grid < 1) grid = 1;
+    // the kernel counts blocks in 32 bits: block + grid stays below 2^31
+    if (nblocks > (int64_t)INT32_MAX - grid) return cudaErrorInvalidValue;
     *grid_out = (int)grid;
     int8_fused_kernel<M, BF16, T><<<(unsigned)grid, T, smem, stream>>>(a, P);
     return cudaGetLastError();
