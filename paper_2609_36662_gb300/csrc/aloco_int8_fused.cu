@@ -34,10 +34,11 @@
 //      block's barrier 1 thread 0 stores the tiles with bulk copies: the M
 //      replica resets are M copies of one tile.  Before barrier 2 of that
 //      block it waits until they have read the tiles.
-// Drift energies: for bf16 with more than 8 workers each block's energies
-// are summed across the warp at once (recursive halving) into fp64 rows;
-// elsewhere fp32 accumulators over up to 8 blocks (at most 64 squares a
-// thread) are reduced worker by worker, in a fixed order.  The squared
+// Drift energies: for bf16 with more than 8 workers and fp32 with 2 or 3,
+// each block's energies are summed across the warp at once (recursive
+// halving) into fp64 rows; elsewhere fp32 accumulators over up to 8 blocks
+// (at most 64 squares a thread) are reduced worker by worker, in a fixed
+// order (see ALOCO_I8_EROW).  The squared
 // decoded means take the second route in every shape.  The arithmetic of
 // every element is the split form's (aloco_int8.cu): the paired operations
 // round each lane as the scalar ones do, so both forms give the same codes,
@@ -312,8 +313,9 @@ __host__ __device__ constexpr bool bf16_one_cta() {
 // element the same way.  Measured on GB300 (4e8 parameters, fraction of the
 // copy peak) against widened pairs: bf16 M = 9 0.956 (0.942), M = 10 0.953
 // (0.920), M = 11 0.935 (0.900), M = 12 0.923 (0.881), M = 16 0.894 (0.863);
-// M = 8 0.865 (0.952).  ALOCO_I8_MIXED = 0 never takes it, 1 always (for
-// bf16), 2 (default) for bf16 with M > 8 (tuning knobs).
+// M = 6 0.956 (0.944); M = 8 0.865 (0.952), M = 5 0.863 (0.937), M = 7 0.866
+// (0.961).  ALOCO_I8_MIXED = 0 never takes it, 1 always (for bf16), 2
+// (default) for bf16 with M > 8 or M = 6 (tuning knobs).
 #ifndef ALOCO_I8_MIXED
 #define ALOCO_I8_MIXED 2
 #endif
@@ -555,14 +557,17 @@ __host__ __device__ constexpr int pow2_at_least(int n) {
 // accumulators over up to 8 blocks reduced worker by worker: bf16 M = 16
 // 0.832 (0.744), M = 12 0.888 (0.861), M = 8 0.947 (0.953); fp32 M = 16
 // (groups, whose energies are reduced per group and block anyway) 0.931
-// (0.932).  Taken for bf16 with M > 8.  ALOCO_I8_EROW = 0 turns it off, 1
-// takes it for every single-group shape (tuning knobs).
+// (0.932); fp32 M = 3 0.958 (0.942), M = 2 0.975 (0.968), bf16 M = 5, 6, 7
+// 0.917, 0.937, 0.937 (0.937, 0.944, 0.961).  Taken for bf16 with M > 8 and
+// fp32 with M = 2, 3.  ALOCO_I8_EROW = 0 turns it off, 1 takes it for every
+// single-group shape (tuning knobs).
 #ifndef ALOCO_I8_EROW
 #define ALOCO_I8_EROW 2
 #endif
 template <int M, bool BF16>
 __host__ __device__ constexpr bool erow() {
-    return ALOCO_I8_EROW == 1 || (ALOCO_I8_EROW == 2 && BF16 && M > 8);
+    return ALOCO_I8_EROW == 1 ||
+           (ALOCO_I8_EROW == 2 && (BF16 ? M > 8 : (M == 2 || M == 3)));
 }
 
 }  // namespace
@@ -591,7 +596,8 @@ __global__ void __launch_bounds__(T, (fused_ctas<M, BF16, T>()))
         ALOCO_I8_NEXT_SMEM == 1 ||
         (ALOCO_I8_NEXT_SMEM == 2 && (fused_ctas<M, BF16, T>() == 1 || (BF16 && M > 8)));
     // bf16 pairs reach the subtraction as raw words (see ALOCO_I8_MIXED)
-    constexpr bool MIX = BF16 && (ALOCO_I8_MIXED == 1 || (ALOCO_I8_MIXED == 2 && M > 8));
+    constexpr bool MIX =
+        BF16 && (ALOCO_I8_MIXED == 1 || (ALOCO_I8_MIXED == 2 && (M > 8 || M == 6)));
     constexpr uint32_t kGVBytes = kI8Block * 4;  // one fp32 array of a block
     constexpr uint32_t kXBytes = kI8Block * ES;  // one replica slice
     // Single buffers suffice: red_w is read between a group's first barrier

@@ -102,9 +102,14 @@ FORMS = {"split": A.PASS_INT8_SPLIT, "fused": A.PASS_INT8_FUSED}
 
 @pytest.mark.parametrize("form", sorted(FORMS))
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
-@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 16])
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 5, 6, 7, 8, 9, 12, 13, 16])
 @pytest.mark.parametrize("parts_name", ["one_part", "ragged", "llama_like"])
 def test_int8_round_matches_oracle(dt, M, parts_name, form):
+    """Every worker count whose fused shape differs: one and two CTAs per
+    SM, theta and v staged or read directly, fp32 worker groups, and for
+    bf16 above 8 workers the mixed-precision subtraction, the energies
+    summed per block over rows padded to a power of two, and (13, 16) the
+    L2 prefetch; every drift energy is checked against the oracle."""
     if form == "fused" and not _fits_fused(dt, M):
         pytest.skip("the fused form holds M <= 16")
     parts = PARTS[parts_name]
