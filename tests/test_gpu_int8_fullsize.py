@@ -1,12 +1,15 @@
 """The INT8-communicated round (App. G.1) at the benchmark's full sizes, in
 the launch configuration bench.py times (AUTO form): the Llama-style 1B set
-with 4 bf16 workers and the 3B set with 8.  Every element of theta', v' and
+with 4 bf16 workers and the 3B set with 8, and the 1B layout with the
+paper's 16 INT8 workers (one CTA per SM, the L2 prefetch of the next block,
+the mixed-precision subtraction and the per-block energy sums).  Every element of theta', v' and
 the replica reset is compared with the oracle's INT8 round, which runs slice
 by slice (whole codec blocks each: the blocks restart at every tensor part)
 on host copies of a device snapshot of the inputs; the slices' sums give the
 whole round's D_t (pre-quantisation pseudo-gradients), ||Dbar||^2 and C_t
 (decoded aggregate), compared at the statistics tolerance; every replica is
 checked on the device to equal theta' rounded to bf16."""
+import dataclasses
 import gc
 
 import pytest
@@ -28,7 +31,12 @@ def _built():
     __graft_entry__.build()
 
 
-@pytest.mark.parametrize("make", [W.llama_1b, W.llama_3b], ids=["llama1b", "llama3b"])
+def _llama_1b_16_workers():
+    return dataclasses.replace(W.llama_1b(), name="llama1b_m16_bf16", M=16)
+
+
+@pytest.mark.parametrize("make", [W.llama_1b, W.llama_3b, _llama_1b_16_workers],
+                         ids=["llama1b", "llama3b", "llama1b_m16"])
 def test_int8_round_full_size_whole_vector(make):
     w = make()
     parts = W.tensor_sizes(w)
