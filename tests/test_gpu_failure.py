@@ -70,8 +70,11 @@ def test_stall_hook_ignored_by_other_rounds():
     assert st["status"] == A.OK and st["pass_used"] == A.PASS_BULK_COPY
 
 
-def test_stalled_int8_fused_block_is_reported_and_the_device_stays_usable():
-    w = W.small(1 << 22, 4, "bf16", seed=5)   # every codec block whole and aligned
+@pytest.mark.parametrize("M", [4, 16], ids=["two_ctas", "one_cta_prefetch"])
+def test_stalled_int8_fused_block_is_reported_and_the_device_stays_usable(M):
+    """M = 4: two CTAs per SM; M = 16: one CTA per SM, which also prefetches
+    the next block into L2 and leaves its place in shared memory."""
+    w = W.small(1 << 22, M, "bf16", seed=5)   # every codec block whole and aligned
     kw = _kw(w)
     fused = lambda: A.default_opts(pass_=A.PASS_INT8_FUSED)
     g, v, xs = gpu_inputs(w)
