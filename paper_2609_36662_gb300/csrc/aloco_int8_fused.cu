@@ -188,7 +188,10 @@ __host__ __device__ constexpr bool fits_two_direct() {
 // two do not fit): bf16 M = 9 0.860 (0.726), M = 10 0.879 (0.738), M = 12
 // 0.835 (0.737); fp32 M = 2 0.979 (0.965), M = 3 0.959 (0.921), M = 4
 // 0.939 (0.903), M = 5 0.926 (0.930).  Staging stays faster for fp32 M = 1
-// (0.984 against 0.931) and bf16 M <= 8 (M = 8: 0.915 against 0.839).
+// (0.984 against 0.931) and bf16 M <= 8 (M = 8: 0.915 against 0.839) except
+// bf16 M = 5: measured again with the current kernel, direct loads gave bf16
+// M = 5 0.953 (0.937) and lost at M = 1..4 and 6..8 (0.83-0.96 against
+// 0.94-0.98), so bf16 M = 5 takes them too.
 // bf16 M >= 13 does not fit two CTAs even so (its replicas alone take more
 // than half an SM).  ALOCO_I8_DIRECT = 0 turns it off, 2 takes it wherever
 // two CTAs fit (tuning knobs).
@@ -199,7 +202,8 @@ template <int M, bool BF16>
 __host__ __device__ constexpr bool direct_gv() {
     if (grouped_direct<M, BF16>()) return true;
     return ALOCO_I8_DIRECT && fused_group<M, BF16>() == M && fits_two_direct<M, BF16>() &&
-           (ALOCO_I8_DIRECT == 2 || !fits_two_staged<M, BF16>() || (!BF16 && M >= 2));
+           (ALOCO_I8_DIRECT == 2 || !fits_two_staged<M, BF16>() || (!BF16 && M >= 2) ||
+            (BF16 && M == 5));
 }
 // theta, v (fp32, unless read directly) and one group's replica slices of
 // one block
