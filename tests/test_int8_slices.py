@@ -78,3 +78,54 @@ def test_a_slice_inside_a_block_would_not_equal_the_whole_round():
     a = O.int8_round(g[:cut], v[:cut], [x[:cut] for x in xs], O.F32, [cut], 0.8, 0.7, 1.0)
     b = O.int8_round(g[cut:], v[cut:], [x[cut:] for x in xs], O.F32, [N - cut], 0.8, 0.7, 1.0)
     assert not np.array_equal(np.concatenate([a["g"], b["g"]]), whole["g"])
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("plant", [None, "theta", "v", "replica"])
+def test_int8_whole_vector_comparison_passes_the_oracle_and_catches_a_plant(dtype, plant):
+    """compare_int8_whole_vector with the oracle's own INT8 round as the
+    outputs: it passes and returns the whole round's statistics; a planted
+    error in theta', v' or replica 0 fails it."""
+    import torch
+
+    from _parity import compare_int8_whole_vector
+    from paper_2609_36662_gb300 import workloads as W
+
+    parts = PART_SETS["ragged"]
+    N, M = sum(parts), 3
+    w = W.small(N, M, dtype, seed=5)
+    rng = np.random.default_rng(6)
+    g = rng.standard_normal(N).astype(np.float32)
+    v = (1e-3 * rng.standard_normal(N)).astype(np.float32)
+    xf = [(g + 1e-3 * rng.standard_normal(N)).astype(np.float32) for _ in range(M)]
+    odt = O.F32 if dtype == "f32" else O.BF16
+    xb = xf if dtype == "f32" else [(x.view(np.uint32) >> 16).astype(np.uint16) for x in xf]
+    corr = O.Correction(1.0, 1.0, 1.0, 1.0, 0.8, 1.0, 0.7, 1.0)
+    whole = O.int8_round(g, v, xb, odt, parts, corr.mu_t, corr.eta_out, corr.inv_norm)
+
+    def tensor(bits):
+        if dtype == "f32":
+            return torch.from_numpy(np.array(bits, np.float32))
+        return torch.from_numpy(bits.view(np.int16).copy()).view(torch.bfloat16)
+
+    g_in, v_in = torch.from_numpy(g), torch.from_numpy(v)
+    x_in = [tensor(x) for x in xb]
+    go = torch.from_numpy(whole["g"].astype(np.float32))
+    vo = torch.from_numpy(whole["v"].astype(np.float32))
+    xo = [tensor(x) for x in whole["x"]]
+    k = 13_000
+    if plant == "theta":
+        go[k] = go[k] * (1 + 1e-3)
+    elif plant == "v":
+        vo[k] = vo[k] * (1 + 1e-3) + 1e-6
+    elif plant == "replica":
+        xo[0][k] = (xo[0][k].float() * 1.01).to(xo[0].dtype)
+    args = (w, parts, g_in, v_in, x_in, go, vo, xo, corr)
+    if plant is None:
+        st = compare_int8_whole_vector(*args, slice_elems=4096, threads=4)
+        assert st["D"] == pytest.approx(whole["D"], rel=1e-12)
+        assert st["C"] == pytest.approx(whole["C"], rel=1e-12)
+        assert st["mean_sq_norm"] == pytest.approx(whole["mean_sq_norm"], rel=1e-12)
+    else:
+        with pytest.raises(AssertionError):
+            compare_int8_whole_vector(*args, slice_elems=4096, threads=4)
